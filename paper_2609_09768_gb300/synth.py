@@ -1,0 +1,173 @@
+"""Seeded synthetic inputs for the selective-recompute prefill.
+
+This module only draws numbers: model shapes, random weights, token ids and the
+chunk layout of a request.  It holds none of the method's arithmetic, so that the
+CUDA path and the CPU oracle can both be fed from it without sharing any code
+that computes the method.
+
+Workload recipe (stand-in for the paper's RULER HQA inputs, Sec. 4 and Tables
+9-10: a long context made of retrieved documents of at most 512 tokens each,
+followed by the question):
+
+* token ids: uniform over the vocabulary;
+* embedding table: N(0, 1), rounded to bf16;
+* linear weights: N(0, 0.02), rounded to bf16 (so both sides read the same values);
+* RMSNorm gains: 1.0;
+* chunks of equal length laid end to end, then a query suffix.
+
+Every tensor is drawn from its own generator, seeded from (seed, layer, name), so
+one layer can be regenerated without drawing the others.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, List, Optional, Sequence
+
+import torch
+
+__all__ = [
+    "ModelShape", "Workload", "SHAPES", "WORKLOADS", "tensor_seed",
+    "make_layer_weights", "make_embed", "make_model", "make_tokens",
+    "chunk_starts_equal", "randn_bf16",
+]
+
+
+@dataclasses.dataclass(frozen=True)
+class ModelShape:
+    """Llama-3.1 decoder shape (hidden, heads, head dim, MLP dim, layers, RoPE)."""
+    hidden: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    mlp_dim: int
+    n_layers: int
+    vocab: int
+    rms_eps: float = 1e-5
+    rope_theta: float = 10000.0
+    rope_llama3: bool = False
+    rs_factor: float = 8.0
+    rs_low: float = 1.0
+    rs_high: float = 4.0
+    rs_orig_ctx: int = 8192
+
+    @property
+    def q_dim(self) -> int:
+        return self.n_q_heads * self.head_dim
+
+    @property
+    def kv_dim(self) -> int:
+        return self.n_kv_heads * self.head_dim
+
+    @property
+    def qkv_dim(self) -> int:
+        return self.q_dim + 2 * self.kv_dim
+
+    def with_layers(self, n_layers: int) -> "ModelShape":
+        return dataclasses.replace(self, n_layers=n_layers)
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    """A request: `n_chunks` chunks of `chunk_len` tokens, a query suffix, ratio r."""
+    name: str
+    shape: ModelShape
+    n_chunks: int
+    chunk_len: int
+    n_query: int
+    r: float = 0.15
+    check_layer: int = 1
+
+    @property
+    def n_ctx(self) -> int:
+        return self.n_chunks * self.chunk_len
+
+    @property
+    def n_total(self) -> int:
+        return self.n_ctx + self.n_query
+
+    def chunk_starts(self) -> List[int]:
+        return chunk_starts_equal(self.n_chunks, self.chunk_len)
+
+
+TINY = ModelShape(hidden=256, n_q_heads=4, n_kv_heads=2, head_dim=64, mlp_dim=688,
+                  n_layers=2, vocab=1024, rms_eps=1e-5, rope_theta=10000.0)
+LLAMA8B = ModelShape(hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128, mlp_dim=14336,
+                     n_layers=32, vocab=128256, rms_eps=1e-5, rope_theta=500000.0,
+                     rope_llama3=True, rs_factor=8.0, rs_low=1.0, rs_high=4.0, rs_orig_ctx=8192)
+
+SHAPES: Dict[str, ModelShape] = {"tiny": TINY, "llama8b": LLAMA8B}
+
+# The single-layer configurations are instantiated with two layers: layer 0 is the
+# full-recompute layer and layer 1 the selective layer under test.
+WORKLOADS: Dict[str, Workload] = {
+    "tiny": Workload("tiny-2L-4x128+32", TINY, 4, 128, 32),
+    "l8b_1layer": Workload("llama8b-2L-8x480+64", LLAMA8B.with_layers(2), 8, 480, 64),
+    "l8b_32k": Workload("llama8b-32L-64x512+128", LLAMA8B, 64, 512, 128),
+    "l8b_124k": Workload("llama8b-32L-242x512+128", LLAMA8B, 242, 512, 128),
+}
+
+
+def tensor_seed(seed: int, layer: int, name: str) -> int:
+    """Deterministic 63-bit seed for one tensor (FNV-1a over the identifiers)."""
+    h = 0xCBF29CE484222325
+    for b in f"{seed}/{layer}/{name}".encode():
+        h ^= b
+        h = (h * 0x100000001B3) & 0xFFFFFFFFFFFFFFFF
+    return h & 0x7FFFFFFFFFFFFFFF
+
+
+def randn_bf16(shape: Sequence[int], seed: int, std: float = 1.0,
+               device: str | torch.device = "cpu") -> torch.Tensor:
+    """N(0, std^2) drawn in fp32 from a generator on `device`, rounded to bf16."""
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    t = torch.randn(*shape, generator=g, device=device, dtype=torch.float32)
+    if std != 1.0:
+        t.mul_(std)
+    return t.to(torch.bfloat16)
+
+
+LAYER_TENSORS = ("w_qkv", "w_o", "w_gate", "w_up", "w_down")
+
+
+def make_layer_weights(shape: ModelShape, layer: int, seed: int = 0,
+                       device: str | torch.device = "cpu") -> Dict[str, torch.Tensor]:
+    """One decoder layer: bf16 matrices (out_features x in_features) and fp32 gains.
+
+    w_qkv rows are [q heads | k heads | v heads], each head `head_dim` rows.
+    """
+    H, F = shape.hidden, shape.mlp_dim
+    dims = {
+        "w_qkv": (shape.qkv_dim, H),
+        "w_o": (H, shape.q_dim),
+        "w_gate": (F, H),
+        "w_up": (F, H),
+        "w_down": (H, F),
+    }
+    w = {n: randn_bf16(dims[n], tensor_seed(seed, layer, n), 0.02, device) for n in LAYER_TENSORS}
+    w["attn_norm"] = torch.ones(H, dtype=torch.float32, device=device)
+    w["mlp_norm"] = torch.ones(H, dtype=torch.float32, device=device)
+    return w
+
+
+def make_embed(shape: ModelShape, seed: int = 0, device: str | torch.device = "cpu") -> torch.Tensor:
+    return randn_bf16((shape.vocab, shape.hidden), tensor_seed(seed, -1, "embed"), 1.0, device)
+
+
+def make_model(shape: ModelShape, seed: int = 0, device: str | torch.device = "cpu") -> dict:
+    return {
+        "layers": [make_layer_weights(shape, l, seed, device) for l in range(shape.n_layers)],
+        "embed": make_embed(shape, seed, device),
+        "final_norm": torch.ones(shape.hidden, dtype=torch.float32, device=device),
+    }
+
+
+def make_tokens(shape: ModelShape, n: int, seed: int = 1, device: str | torch.device = "cpu") -> torch.Tensor:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(tensor_seed(seed, -2, "tokens"))
+    return torch.randint(0, shape.vocab, (n,), generator=g, dtype=torch.int64).to(torch.int32).to(device)
+
+
+def chunk_starts_equal(n_chunks: int, chunk_len: int) -> List[int]:
+    return [c * chunk_len for c in range(n_chunks + 1)]
+
