@@ -1,0 +1,282 @@
+/*
+ * kvblend.h - C ABI of the GB300 selective-recompute prefill library (libkvblend.so).
+ *
+ * The library computes the prefill that runs after per-chunk KV caches are
+ * concatenated (the CacheBlend-style selective recompute combined with a
+ * concatenation-aware model in the paper "Fine-Tuning a KV Cache
+ * Concatenation-Aware Model or Recomputing KV Caches? Why Not Both?"):
+ * position re-alignment of each chunk's cached keys (Sec. 3.4, Sec. 4), full
+ * causal recompute of layer 0 (Sec. 4), per-token key deviation and top-k
+ * selection at ratio r (Sec. 2, Sec. 3.2), and, in every later layer, the
+ * recompute of the selected rows with attention over the whole blended cache
+ * under a causal mask (Sec. 4, Limitations).
+ *
+ * Conventions shared by every call
+ *  - Pointers named *_host are host memory; every other data pointer is device
+ *    memory of the current CUDA device.  The caller owns all buffers; the library
+ *    never allocates or frees device memory.  Scratch memory comes from a caller
+ *    workspace whose size kvb_workspace_size() / kvb_hkvd_workspace_size() give.
+ *  - bf16 tensors are passed as uint16_t* (raw bfloat16 bits); fp32 as float*.
+ *  - All device pointers must be 16-byte aligned.  Matrices are row-major and dense.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Every call is asynchronous on that stream and enqueues no host synchronisation,
+ *    except kvb_device_status(), which synchronises the stream.
+ *  - Return value: KVB_OK, or an error code for argument validation (before any
+ *    launch) or a CUDA launch error.  kvb_last_error() returns a message for the
+ *    last failing call on the calling thread.  Errors detected on the device
+ *    (a bounded wait that ran out) are recorded in the workspace status word and
+ *    read with kvb_device_status().  The word is the first 4 bytes of a workspace:
+ *    zero the workspace's first 256 bytes once before its first use; calls never
+ *    clear it, kvb_device_status() clears it after reading.
+ *
+ * Model layout (Llama-3.1 decoder, Sec. 4): hidden H, Hq query heads, Hkv kv heads,
+ * head dim D in {64, 128}, MLP dim F, Hq % Hkv == 0 and 128 % (Hq/Hkv) == 0.
+ *  - KV cache of one layer: [n_rows][Hkv][D] bf16 for K and for V; a multi-layer
+ *    cache is n_layers such blocks back to back.  Row t of the blended cache holds
+ *    token t of the concatenated sequence (global position t).
+ *  - RoPE is rotate-half (dimension i pairs with i + D/2); tables hold
+ *    cos/sin(pos * w_i) in fp32, [max_pos][D/2], computed in double precision.
+ */
+#ifndef KVBLEND_H
+#define KVBLEND_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum kvb_status {
+    KVB_OK = 0,
+    KVB_ERR_INVALID_ARG = 1,   /* a pointer, size or shape the call cannot accept       */
+    KVB_ERR_UNSUPPORTED = 2,   /* valid in principle but not built (e.g. head_dim 96)   */
+    KVB_ERR_CUDA = 3,          /* a CUDA runtime/driver call or a launch failed         */
+    KVB_ERR_TIMEOUT = 4,       /* device side: a bounded wait in a kernel ran out       */
+    KVB_ERR_WORKSPACE = 5      /* workspace missing or smaller than required            */
+} kvb_status;
+
+/* Model shape and RoPE settings (Llama 3.1 frequency scaling when rope_llama3 != 0:
+ * factor rs_factor, low/high frequency factors rs_low/rs_high, original context
+ * rs_orig_ctx). */
+typedef struct kvb_config {
+    int32_t hidden, n_q_heads, n_kv_heads, head_dim, mlp_dim, n_layers, vocab;
+    float rms_eps;
+    float rope_theta;
+    int32_t rope_llama3;
+    float rs_factor, rs_low, rs_high;
+    int32_t rs_orig_ctx;
+} kvb_config;
+
+/* Device pointers of one decoder layer.  Linear weights are [out][in] bf16:
+ * w_qkv [(Hq+2Hkv)D][H] (rows: q heads, then k heads, then v heads), w_o [H][Hq D],
+ * w_gate and w_up [F][H], w_down [H][F]; norm gains are fp32 [H]. */
+typedef struct kvb_layer_weights {
+    const float* attn_norm;
+    const uint16_t* w_qkv;
+    const uint16_t* w_o;
+    const float* mlp_norm;
+    const uint16_t* w_gate;
+    const uint16_t* w_up;
+    const uint16_t* w_down;
+} kvb_layer_weights;
+
+/* Whole model: `layers` is a HOST array of n_layers entries; embed is [vocab][H] bf16,
+ * final_norm [H] fp32 (device). */
+typedef struct kvb_model {
+    const kvb_layer_weights* layers;
+    const uint16_t* embed;
+    const float* final_norm;
+} kvb_model;
+
+/* RoPE tables in device memory, fp32 [max_pos][D/2] each. */
+typedef struct kvb_rope_table {
+    const float* cos;
+    const float* sin;
+    int64_t max_pos;
+} kvb_rope_table;
+
+/* Multi-layer KV cache: k and v are [n_layers][n_rows][Hkv][D] bf16. */
+typedef struct kvb_kv_cache {
+    uint16_t* k;
+    uint16_t* v;
+    int64_t n_rows;
+    int32_t n_layers;
+} kvb_kv_cache;
+
+/* Stage times of one prefill in milliseconds (CUDA events on the call's stream). */
+typedef struct kvb_timings {
+    float total_ms;
+    float realign_ms;     /* merge + position re-alignment of the chunk caches      */
+    float dense_ms;       /* layers before the check layer, all rows (layer 0)       */
+    float select_ms;      /* check-layer keys, deviation and top-k                    */
+    float selective_ms;   /* selective layers over the recomputed rows                */
+    float final_ms;       /* final RMSNorm of the query rows                          */
+    int64_t n_selected;   /* k = number of recomputed context rows                   */
+    int64_t n_rows;       /* m = k + n_query                                          */
+} kvb_timings;
+
+/* ------------------------------------------------------------------ status */
+
+/* Static text for a status code. */
+const char* kvb_status_string(kvb_status s);
+/* Message of the last failing call on this thread ("" if none).  Thread-local. */
+const char* kvb_last_error(void);
+/* Library ABI version (major * 100 + minor). */
+int32_t kvb_version(void);
+
+/* ------------------------------------------------------------------ RoPE */
+
+/* Fill HOST tables cos_host/sin_host, each [max_pos][D/2] fp32, with cos/sin of
+ * pos * w_i for pos < max_pos (w_i = theta^(-2i/D), Llama 3.1 scaling if enabled;
+ * Sec. 4 asks for the position adjustment in float32 - angles are formed in double
+ * and rounded once).  Pure host call.  Errors: INVALID_ARG for NULL pointers,
+ * max_pos < 1 or an unsupported head_dim. */
+kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos,
+                               float* cos_host, float* sin_host);
+
+/* ------------------------------------------------------------------ steps */
+
+/* Merge + position re-alignment (Sec. 3.4 "merged into one, followed by position
+ * adjustment"; PIE, Sec. 2).  For layers [layer_begin, layer_end) and every context
+ * row t < n_ctx in chunk c (chunk_start[c] <= t < chunk_start[c+1]):
+ *   k_dst[l][t] = R(chunk_start[c]) k_src[l][t]   (rotation of every head's pairs by
+ *                                                  the chunk offset, fp32 math)
+ *   v_dst[l][t] = v_src[l][t]                     (skipped when v_src == v_dst or NULL)
+ * k_src/v_src are [n_layers][src_rows][Hkv][D] with keys rotated at chunk-local
+ * positions; k_dst/v_dst are [n_layers][dst_rows][Hkv][D].  In place is allowed
+ * (k_src == k_dst, src_rows == dst_rows).  chunk_start: DEVICE int32 [n_chunks+1],
+ * ascending, chunk_start[0] == 0, chunk_start[n_chunks] == n_ctx.  The rope table
+ * must cover max_pos > chunk_start[n_chunks-1].  Errors: INVALID_ARG. */
+kvb_status kvb_rope_realign(const kvb_config* cfg, const kvb_rope_table* rope,
+                            const uint16_t* k_src, const uint16_t* v_src, int64_t src_rows,
+                            uint16_t* k_dst, uint16_t* v_dst, int64_t dst_rows,
+                            int32_t layer_begin, int32_t layer_end,
+                            const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
+                            void* stream);
+
+/* Workspace bytes kvb_hkvd_select needs for n_ctx rows. */
+size_t kvb_hkvd_workspace_size(int64_t n_ctx);
+
+/* HKVD deviation and top-k (Sec. 2 on CacheBlend, Sec. 3.2: tokens whose keys
+ * deviate most, by squared key difference, are recomputed):
+ *   dev_out[i] = sum over kv heads and dims of (k_fresh[i] - k_cached[i])^2   (fp32)
+ *   sel_out    = the k indices with the largest dev, ties to the lower index,
+ *                written in ascending order.
+ * k_fresh row i at k_fresh + i*ld_fresh, k_cached row i at k_cached + i*ld_cached
+ * (elements), kv_dim elements per row (multiple of 8).  0 <= k <= n_ctx.
+ * dev_out: [n_ctx] fp32 (required); sel_out: [k] int32.  Workspace: at least
+ * kvb_hkvd_workspace_size(n_ctx) bytes, 256-byte aligned.  Errors: INVALID_ARG,
+ * WORKSPACE. */
+kvb_status kvb_hkvd_select(const uint16_t* k_fresh, int64_t ld_fresh,
+                           const uint16_t* k_cached, int64_t ld_cached,
+                           int64_t n_ctx, int32_t kv_dim, int64_t k,
+                           int32_t* sel_out, float* dev_out,
+                           void* ws, size_t ws_bytes, void* stream);
+
+/* Gather + RMSNorm + QKV projection + RoPE for m rows (the per-row front half of a
+ * decoder layer, Sec. 4 model):
+ *   a[r]   = RMSNorm(x[row_idx[r]]) * attn_norm          (x: fp32 [*][H]; row_idx NULL = r)
+ *   q[r]   = RoPE(a[r] W_q^T, rope_pos[r])  -> q_out [m][Hq D] bf16
+ *   k[r]   = RoPE(a[r] W_k^T, rope_pos[r])  -> k_out row kv_dst[r] (or r), [*][Hkv D] bf16
+ *   v[r]   = a[r] W_v^T                     -> v_out row kv_dst[r] (or r)
+ * Passing a cache layer as k_out/v_out with kv_dst = the rows' cache indices fuses the
+ * KV scatter.  rope_pos: [m] int32 (< rope->max_pos).  Uses tcgen05 tensor cores
+ * (bf16 in, fp32 accumulate).  Workspace >= kvb_workspace_size(cfg, m).  Errors:
+ * INVALID_ARG, WORKSPACE, UNSUPPORTED. */
+kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights* w,
+                                  const kvb_rope_table* rope,
+                                  const float* x, const int32_t* row_idx,
+                                  const int32_t* rope_pos, int64_t m,
+                                  uint16_t* q_out, uint16_t* k_out, uint16_t* v_out,
+                                  const int32_t* kv_dst,
+                                  void* ws, size_t ws_bytes, void* stream);
+
+/* KV scatter (Sec. 3.4: recomputed entries replace the cached ones): for r < m,
+ *   k_dst[dst_idx[r]] = k_rows[r], v_dst[dst_idx[r]] = v_rows[r]   (kv_dim elements)
+ * dst_idx values must be distinct and < n_dst_rows (bit copy, order irrelevant).
+ * Errors: INVALID_ARG. */
+kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows,
+                          const int32_t* dst_idx, int64_t m, int32_t kv_dim,
+                          uint16_t* k_dst, uint16_t* v_dst, int64_t n_dst_rows,
+                          void* stream);
+
+/* Sparse-query causal GQA attention (Sec. 4: recompute with an attention mask;
+ * Limitations 1: selected query rows attending the whole cache, causally):
+ *   out[r, j] = sum_{t = lo_r}^{hi_r} softmax_t(q[r, j] . K[t, g] / sqrt(D)) V[t, g],
+ *   g = j / (Hq/Hkv), hi_r = q_idx[r], lo_r = kv_lo ? kv_lo[r] : 0.
+ * q: [m][Hq][D] bf16 (rotated); q_idx: [m] int32, ascending, < n_kv; kv_lo: [m] or
+ * NULL; k_cache/v_cache: one layer, [n_kv][Hkv][D] bf16; out: [m][Hq D] bf16.
+ * tcgen05 tensor cores, fp32 softmax.  Errors: INVALID_ARG, UNSUPPORTED. */
+kvb_status kvb_sparse_query_attn(const kvb_config* cfg, const uint16_t* q,
+                                 const int32_t* q_idx, const int32_t* kv_lo, int64_t m,
+                                 const uint16_t* k_cache, const uint16_t* v_cache, int64_t n_kv,
+                                 uint16_t* out, void* ws, size_t ws_bytes, void* stream);
+
+/* Back half of a decoder layer on m rows (Sec. 4 model):
+ *   x[r] += attn[r] W_o^T;  x[r] += W_down (silu(W_gate n) * (W_up n)),  n = RMSNorm(x[r]) * mlp_norm
+ * attn: [m][Hq D] bf16; x: [m][H] fp32, updated in place.  Workspace >=
+ * kvb_workspace_size(cfg, m).  Errors: INVALID_ARG, WORKSPACE. */
+kvb_status kvb_mlp_rows(const kvb_config* cfg, const kvb_layer_weights* w,
+                        const uint16_t* attn, int64_t m, float* x,
+                        void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------ whole prefill */
+
+/* Workspace bytes for a prefill (or a single step) over up to n_rows rows. */
+kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* bytes);
+
+/* Selective-recompute prefill over concatenated per-chunk caches (the whole path):
+ *  1. merge + re-align the chunk caches of layers >= check_layer into `cache`
+ *     (rows [0, n_ctx) of each layer);
+ *  2. layers < check_layer (layer 0 at least): all n = n_ctx + n_query rows, causal;
+ *  3. check layer: fresh keys of all context rows at global positions, deviation
+ *     against the re-aligned cache, top-k with k = floor(r * n_ctx) (or the forced set);
+ *  4. layers >= check_layer: rows S = selected context rows + the n_query query rows,
+ *     K/V scattered into the cache before attention over the whole cache;
+ *  5. final RMSNorm of the query rows -> final_hidden [n_query][H] fp32.
+ * k_chunks/v_chunks: [n_layers][n_ctx][Hkv][D] bf16, each chunk's cache at chunk-local
+ * positions (read only).  cache: output blended cache with n_rows >= n_ctx + n_query.
+ * token_ids: DEVICE int32 [n_ctx + n_query]; chunk_start: DEVICE int32 [n_chunks+1]
+ * with chunk_start[n_chunks] == n_ctx.  r in [0, 1]; 1 <= check_layer <= n_layers
+ * (check_layer == n_layers means every layer is dense).  forced_sel: DEVICE int32
+ * [forced_k] ascending distinct context indices, or NULL.  sel_out: DEVICE int32 [n_ctx]
+ * or NULL (receives the k chosen indices).  t: HOST timings or NULL (timing adds
+ * events but no synchronisation until the call returns; with t != NULL the call
+ * synchronises the stream once at the end to read the events).  r == 1 computes
+ * the dense prefill of every layer.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
+kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
+                                 const kvb_rope_table* rope,
+                                 const uint16_t* k_chunks, const uint16_t* v_chunks,
+                                 kvb_kv_cache* cache,
+                                 const int32_t* token_ids, const int32_t* chunk_start,
+                                 int32_t n_chunks, int64_t n_ctx, int64_t n_query,
+                                 float r, int32_t check_layer,
+                                 const int32_t* forced_sel, int64_t forced_k,
+                                 float* final_hidden, int32_t* sel_out,
+                                 kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
+
+/* Dense causal prefill of n rows through every layer (the r = 1 comparator, Sec. 4;
+ * also the per-chunk isolated prefill that produces chunk caches):
+ *   row t attends cache rows [kv_lo[t], t] (kv_lo NULL = 0) with RoPE at rope_pos[t]
+ *   (NULL = t).  With kv_lo = chunk start and rope_pos = t - chunk start every chunk
+ *   is prefilled alone at chunk-local positions.
+ * Writes every layer's K/V into cache rows [0, n) and, if final_hidden != NULL, the
+ * final RMSNorm of the last n_out rows to final_hidden [n_out][H].  Errors as above. */
+kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
+                            const kvb_rope_table* rope, kvb_kv_cache* cache,
+                            const int32_t* token_ids, int64_t n,
+                            const int32_t* rope_pos, const int32_t* kv_lo,
+                            float* final_hidden, int64_t n_out,
+                            kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronise `stream`, then read and clear the device status word that kernels using
+ * workspace `ws` write when a bounded wait runs out.  *code_out receives KVB_OK or
+ * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */
+kvb_status kvb_device_status(void* ws, size_t ws_bytes, void* stream, int32_t* code_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVBLEND_H */

@@ -1,0 +1,355 @@
+// Sparse-query causal GQA flash attention on the 5th-generation tensor cores.
+//
+// Each CTA owns one (block of query rows, kv head) unit.  The Hq/Hkv query heads
+// that share kv head g are packed with 128/(Hq/Hkv) query rows into the 128 rows
+// of one MMA tile (lane = row_in_block * G + head_in_group), so every K/V tile
+// loaded serves all G heads.  Row r attends cache rows [lo_r, hi_r] where hi_r is
+// the row's own cache index: this one predicate covers the sparse recompute rows
+// of the selective layers, the dense causal prefill and the block-diagonal
+// per-chunk prefill.
+//
+// Pipeline per key tile j (128 keys):
+//   TMA warp   : K_j, V_j into 2-deep rings (128-byte swizzle)
+//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=128, K=16 steps);
+//                after the softmax of tile j-1, O += P_{j-1} V_{j-1} (V as an
+//                MN-major operand, O accumulated in TMEM)
+//   4 softmax warps (thread = row): read S_j from TMEM, mask, online softmax with
+//                a lazily updated running max (O is rescaled only when the max
+//                grows by more than 2^8), write P_j (bf16) to swizzled smem.
+// Lazy rescaling keeps the result exact: every term uses the same reference max
+// as the running sum it is divided by.
+#include <float.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace kvb {
+namespace {
+
+constexpr int THREADS = 192;
+constexpr int KT_ROWS = 128;                 // keys per tile
+constexpr uint32_t TMEM_COLS = 512;
+constexpr float RESCALE_LOG2 = 8.0f;
+
+template <int D>
+struct Smem {
+    static constexpr int CHUNK = 128 * 128;              // 128 rows x 128 bytes
+    static constexpr int Q_BYTES = (D / 64) * CHUNK;
+    static constexpr int KV_BYTES = (D / 64) * CHUNK;    // one K or V tile
+    static constexpr int P_BYTES = 2 * CHUNK;            // 128 rows x 128 keys bf16
+    static constexpr int OFF_Q = 0;
+    static constexpr int OFF_K = OFF_Q + Q_BYTES;
+    static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
+    static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
+    static constexpr int OFF_BAR = OFF_P + P_BYTES;
+    static constexpr int TOTAL = OFF_BAR + 256 + 1024;
+};
+
+template <int D>
+__global__ void __launch_bounds__(THREADS, 1)
+attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+            const __grid_constant__ CUtensorMap tmV, const AttnParams p, int num_blocks) {
+    using S = Smem<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
+    uint64_t* q_full = bars + 0;
+    uint64_t* k_full = bars + 1;     // [2]
+    uint64_t* k_empty = bars + 3;    // [2]
+    uint64_t* v_full = bars + 5;     // [2]
+    uint64_t* v_empty = bars + 7;    // [2]
+    uint64_t* s_full = bars + 9;     // [2]
+    uint64_t* s_free = bars + 11;    // [2]
+    uint64_t* p_full = bars + 13;
+    uint64_t* pv_done = bars + 14;
+    uint64_t* drain = bars + 15;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* red = reinterpret_cast<int*>(tmem_slot + 2);   // lo_min, hi_max, hi_min, lo_max
+
+    const uint32_t warp = warp_id(), lane = lane_id();
+    const int G = p.Hq / p.Hkv;
+    const int RPB = 128 / G;
+    const int blk = num_blocks - 1 - (int)(blockIdx.x / p.Hkv);   // heaviest rows first
+    const int g = (int)(blockIdx.x % p.Hkv);
+    const int64_t r0 = (int64_t)blk * RPB;
+
+    if (threadIdx.x == 0) {
+        mbar_init(q_full, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&k_full[b], 1); mbar_init(&k_empty[b], 1);
+            mbar_init(&v_full[b], 1); mbar_init(&v_empty[b], 1);
+            mbar_init(&s_full[b], 1); mbar_init(&s_free[b], 4);
+        }
+        mbar_init(p_full, 4);
+        mbar_init(pv_done, 1);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        red[0] = INT_MAX; red[1] = -1; red[2] = INT_MAX; red[3] = -1;
+        fence_mbar_init();
+    }
+    if (warp == 1) { tmem_alloc(tmem_slot, TMEM_COLS); tmem_relinquish(); }
+    __syncthreads();
+
+    // this thread's row (softmax warps); key range of the whole block
+    const uint32_t quarter = warp & 3;
+    const int L = (int)(quarter * 32 + lane);
+    const int64_t row = r0 + L / G;
+    const int head = g * G + L % G;
+    const bool valid = warp >= 2 && row < p.m;
+    int hi = -1, lo = 0;
+    if (valid) {
+        hi = p.q_idx[row];
+        lo = p.kv_lo ? p.kv_lo[row] : 0;
+        atomicMin(&red[0], lo);
+        atomicMax(&red[1], hi);
+        atomicMin(&red[2], hi);
+        atomicMax(&red[3], lo);
+    }
+    if (warp == 0 && lane == 0) { prefetch_tmap(&tmQ); prefetch_tmap(&tmK); prefetch_tmap(&tmV); }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const int lo_min = red[0], hi_max = red[1], hi_min = red[2], lo_max = red[3];
+    const int t_begin = lo_min / KT_ROWS;
+    const int n_tiles = hi_max < 0 ? 0 : hi_max / KT_ROWS + 1 - t_begin;
+
+    uint8_t* sQ = smem + S::OFF_Q;
+    uint8_t* sK = smem + S::OFF_K;
+    uint8_t* sV = smem + S::OFF_V;
+    uint8_t* sP = smem + S::OFF_P;
+
+    if (warp == 0) {
+        if (lane == 0 && n_tiles > 0) {
+            // ------------------------------------------------ TMA producer
+            mbar_expect_tx(q_full, S::Q_BYTES);
+#pragma unroll
+            for (int c = 0; c < D / 64; ++c) tma_load_3d(sQ + c * S::CHUNK, &tmQ, q_full, c * 64, g * G, (int)r0);
+            int issued_k = 0, issued_v = 0;
+            for (int j = 0; j < n_tiles; ++j) {
+                const int b = j & 1;
+                const uint32_t ph = (j >> 1) & 1;
+                const int y = (t_begin + j) * KT_ROWS;
+                if (!mbar_wait(&k_empty[b], ph ^ 1, abort_flag, p.status)) break;
+                mbar_expect_tx(&k_full[b], S::KV_BYTES);
+#pragma unroll
+                for (int c = 0; c < D / 64; ++c)
+                    tma_load_2d(sK + b * S::KV_BYTES + c * S::CHUNK, &tmK, &k_full[b], g * D + c * 64, y);
+                issued_k = j + 1;
+                if (!mbar_wait(&v_empty[b], ph ^ 1, abort_flag, p.status)) break;
+                mbar_expect_tx(&v_full[b], S::KV_BYTES);
+#pragma unroll
+                for (int c = 0; c < D / 64; ++c)
+                    tma_load_2d(sV + b * S::KV_BYTES + c * S::CHUNK, &tmV, &v_full[b], g * D + c * 64, y);
+                issued_v = j + 1;
+            }
+            // on the abort path, let the loads already issued land before exiting
+            if (*abort_flag) {
+                const uint64_t t0 = globaltimer();
+                for (int j = (issued_k > 2 ? issued_k - 2 : 0); j < issued_k; ++j)
+                    while (!mbar_try_wait(&k_full[j & 1], (j >> 1) & 1) && globaltimer() - t0 < 1000000ull) {}
+                for (int j = (issued_v > 2 ? issued_v - 2 : 0); j < issued_v; ++j)
+                    while (!mbar_try_wait(&v_full[j & 1], (j >> 1) & 1) && globaltimer() - t0 < 1000000ull) {}
+                while (!mbar_try_wait(q_full, 0) && globaltimer() - t0 < 1000000ull) {}
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && n_tiles > 0) {
+            // ------------------------------------------------ MMA issuer
+            constexpr uint32_t IDESC_S = idesc_bf16(128, KT_ROWS, false);
+            constexpr uint32_t IDESC_O = idesc_bf16(128, D, true);
+            const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(sK), v0 = smem_u32(sV), p0 = smem_u32(sP);
+            bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
+            tc_fence_after();
+            for (int j = 0; ok && j <= n_tiles; ++j) {
+                if (j < n_tiles) {
+                    const int b = j & 1;
+                    if (!mbar_wait(&k_full[b], (j >> 1) & 1, abort_flag, p.status)) break;
+                    if (j >= 2 && !mbar_wait(&s_free[b], ((j - 2) >> 1) & 1, abort_flag, p.status)) break;
+                    tc_fence_after();
+                    const uint32_t kb = k0 + b * S::KV_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        const uint32_t off = (kk >> 2) * S::CHUNK + (kk & 3) * 32;
+                        mma_bf16_ss(tmem_base + b * KT_ROWS, sdesc_sw128(q0 + off, 16, 1024),
+                                    sdesc_sw128(kb + off, 16, 1024), IDESC_S, kk > 0);
+                    }
+                    mma_commit(&k_empty[b]);
+                    mma_commit(&s_full[b]);
+                }
+                if (j >= 1) {
+                    const int i = j - 1, bi = i & 1;
+                    if (!mbar_wait(p_full, i & 1, abort_flag, p.status)) break;
+                    if (!mbar_wait(&v_full[bi], (i >> 1) & 1, abort_flag, p.status)) break;
+                    tc_fence_after();
+                    const uint32_t vb = v0 + bi * S::KV_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < KT_ROWS / 16; ++kk) {
+                        const uint32_t offp = (kk >> 2) * S::CHUNK + (kk & 3) * 32;
+                        mma_bf16_ss(tmem_base + 2 * KT_ROWS, sdesc_sw128(p0 + offp, 16, 1024),
+                                    sdesc_sw128(vb + kk * 16 * 128, S::CHUNK, 1024), IDESC_O, (i > 0) || (kk > 0));
+                    }
+                    mma_commit(&v_empty[bi]);
+                    mma_commit(pv_done);
+                }
+            }
+            mma_commit(drain);
+            const uint64_t t0 = globaltimer();
+            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+        }
+    } else if (n_tiles > 0) {
+        // ---------------------------------------------------- softmax warps (2..5)
+        const float sl2 = p.scale_log2;
+        const uint32_t lane_addr = (quarter * 32u) << 16;
+        float m_run = -INFINITY, l_run = 0.f;
+        bool ok = true;
+        for (int j = 0; j < n_tiles; ++j) {
+            const int b = j & 1;
+            if (!mbar_wait_warp(&s_full[b], (j >> 1) & 1, abort_flag, p.status)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t s[KT_ROWS];
+#pragma unroll
+            for (int c = 0; c < KT_ROWS / 32; ++c) tmem_ld32(tmem_base + lane_addr + b * KT_ROWS + c * 32, s + c * 32);
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_free[b]);
+
+            const int key0 = (t_begin + j) * KT_ROWS;
+            const bool full_vis = key0 >= lo_max && key0 + KT_ROWS - 1 <= hi_min;
+            float mt = -INFINITY;
+            if (full_vis) {
+#pragma unroll
+                for (int c = 0; c < KT_ROWS; ++c) mt = fmaxf(mt, __uint_as_float(s[c]));
+            } else {
+#pragma unroll
+                for (int c = 0; c < KT_ROWS; ++c) {
+                    const int key = key0 + c;
+                    float v = __uint_as_float(s[c]);
+                    if (key > hi || key < lo) v = -INFINITY;
+                    s[c] = __float_as_uint(v);
+                    mt = fmaxf(mt, v);
+                }
+            }
+            const float m_new = fmaxf(m_run, mt);
+            const bool resc = (m_new - m_run) * sl2 > RESCALE_LOG2;   // false when both are -inf
+            float alpha = 1.f;
+            if (resc) {
+                alpha = fast_exp2((m_run - m_new) * sl2);           // 0 when m_run = -inf
+                l_run *= alpha;
+                m_run = m_new;
+            }
+            const float mref = (m_run == -INFINITY) ? 0.f : m_run * sl2;
+            uint32_t pk[KT_ROWS / 2];
+            float lsum = 0.f;
+#pragma unroll
+            for (int c = 0; c < KT_ROWS; c += 2) {
+                const float e0 = fast_exp2(fmaf(__uint_as_float(s[c]), sl2, -mref));
+                const float e1 = fast_exp2(fmaf(__uint_as_float(s[c + 1]), sl2, -mref));
+                lsum += e0 + e1;
+                pk[c / 2] = pack_bf16(e0, e1);
+            }
+            l_run += lsum;
+
+            if (j >= 1) {
+                if (!mbar_wait_warp(pv_done, (j - 1) & 1, abort_flag, p.status)) { ok = false; break; }
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, resc)) {
+                    const uint32_t oaddr = tmem_base + lane_addr + 2 * KT_ROWS;
+#pragma unroll 1
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(oaddr + c * 32, o);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        tmem_st32(oaddr + c * 32, o);
+                    }
+                    tmem_st_wait();
+                }
+            }
+            // P row L into the 128-byte-swizzled K-major operand layout
+#pragma unroll
+            for (int u = 0; u < KT_ROWS / 8; ++u) {
+                const int chunk = u >> 3, uu = u & 7;
+                uint8_t* dst = sP + chunk * S::CHUNK + (L >> 3) * 1024 + (L & 7) * 128 + ((uu ^ (L & 7)) << 4);
+                *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+            }
+            fence_async_smem();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(p_full);
+        }
+        if (ok && mbar_wait_warp(pv_done, (n_tiles - 1) & 1, abort_flag, p.status)) {
+            tc_fence_after();
+            const uint32_t oaddr = tmem_base + lane_addr + 2 * KT_ROWS;
+            const float inv = (l_run > 0.f) ? 1.f / l_run : 0.f;
+            uint16_t* dst = p.out + row * (int64_t)(p.Hq * D) + (int64_t)head * D;
+#pragma unroll 1
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(oaddr + c * 32, o);
+                tmem_ld_wait();
+                if (valid) {
+                    uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        const int e = q4 * 8;
+                        d4[q4] = make_uint4(pack_bf16(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv),
+                                            pack_bf16(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv),
+                                            pack_bf16(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
+                                            pack_bf16(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, TMEM_COLS);
+    }
+}
+
+template <int D>
+kvb_status run(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v, const AttnParams& p, int nb,
+               cudaStream_t st) {
+    static bool attr_set = false;
+    auto kern = attn_kernel<D>;
+    if (!attr_set) {
+        kvb_status s = cuda_ok(
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<D>::TOTAL), "attn smem");
+        if (s != KVB_OK) return s;
+        attr_set = true;
+    }
+    const int64_t grid = (int64_t)nb * p.Hkv;
+    kern<<<(unsigned)grid, THREADS, Smem<D>::TOTAL, st>>>(q, k, v, p, nb);
+    return cuda_ok(cudaGetLastError(), "attention launch");
+}
+
+}  // namespace
+
+kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
+                       cudaStream_t st) {
+    if (p.m <= 0) return KVB_OK;
+    if (p.D != 64 && p.D != 128) return fail(KVB_ERR_UNSUPPORTED, "attention: head_dim %d not built", p.D);
+    if (p.Hkv <= 0 || p.Hq % p.Hkv || 128 % (p.Hq / p.Hkv))
+        return fail(KVB_ERR_UNSUPPORTED, "attention: Hq/Hkv must divide 128");
+    const int G = p.Hq / p.Hkv, RPB = 128 / G;
+    CUtensorMap tq, tk, tv;
+    kvb_status s = make_tmap_3d(&tq, q, (uint64_t)p.D, (uint64_t)p.Hq, (uint64_t)p.m, 64, (uint32_t)G, (uint32_t)RPB);
+    if (s != KVB_OK) return s;
+    const uint64_t kvd = (uint64_t)p.Hkv * p.D;
+    s = make_tmap_2d(&tk, k_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
+    if (s != KVB_OK) return s;
+    s = make_tmap_2d(&tv, v_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
+    if (s != KVB_OK) return s;
+    const int64_t nb = (p.m + RPB - 1) / RPB;
+    if (nb * p.Hkv > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "attention: too many rows");
+    return p.D == 128 ? run<128>(tq, tk, tv, p, (int)nb, st) : run<64>(tq, tk, tv, p, (int)nb, st);
+}
+
+}  // namespace kvb

@@ -1,0 +1,114 @@
+// Host-side internals shared by the translation units of libkvblend.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kvblend.h"
+
+namespace kvb {
+
+// Record a message for kvb_last_error() and return the status.
+kvb_status fail(kvb_status s, const char* fmt, ...);
+// KVB_OK, or KVB_ERR_CUDA with the CUDA error text.
+kvb_status cuda_ok(cudaError_t e, const char* what);
+int num_sms();
+bool aligned16(const void* p);
+
+// Tensor map for a row-major bf16 matrix [rows][cols] (row stride ld elements),
+// box [box_rows][box_cols], 128-byte swizzle.
+kvb_status make_tmap_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld,
+                        uint32_t box_cols, uint32_t box_rows);
+// Tensor map over [d2][d1][d0] bf16 (dense), box [b2][b1][b0], 128-byte swizzle.
+kvb_status make_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                        uint32_t b0, uint32_t b1, uint32_t b2);
+
+// ---------------------------------------------------------------- GEMM (tcgen05)
+
+enum GemmEpi : int { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2 };
+
+struct GemmParams {
+    int64_t M, N, K;
+    int epi;
+    // EPI_QKV: output column c of this GEMM is column col_base + c of [q | k | v]
+    int col_base, q_dim, kv_dim, head_dim;
+    uint16_t* q_out;
+    uint16_t* k_out;
+    uint16_t* v_out;
+    const int32_t* kv_dst;
+    const int32_t* rope_pos;
+    const float* cos_t;
+    const float* sin_t;
+    // EPI_RESID: x[r][c] += acc
+    float* x;
+    int64_t ldx;
+    // EPI_SWIGLU: out[r][c] = silu(gate) * up
+    uint16_t* out;
+    int64_t ldo;
+    int* status;
+};
+
+// C = A B^T with A [M][K] (row stride lda), B [N][K] (row stride ldb); for EPI_SWIGLU
+// B is the gate matrix and B2 the up matrix, both [N][K].
+kvb_status launch_gemm(const GemmParams& p, const uint16_t* A, int64_t lda, const uint16_t* B, int64_t ldb,
+                       const uint16_t* B2, cudaStream_t st);
+
+// ---------------------------------------------------------------- attention (tcgen05)
+
+struct AttnParams {
+    const int32_t* q_idx;
+    const int32_t* kv_lo;
+    int64_t m, n_kv;
+    int Hq, Hkv, D;
+    uint16_t* out;
+    float scale_log2;
+    int* status;
+};
+kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
+                       cudaStream_t st);
+
+// ---------------------------------------------------------------- memory-bound kernels
+
+kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv, const uint16_t* k_src,
+                          const uint16_t* v_src, int64_t src_layer_stride, uint16_t* k_dst, uint16_t* v_dst,
+                          int64_t dst_layer_stride, int n_layers, const int32_t* chunk_start, int n_chunks,
+                          int64_t n_ctx, cudaStream_t st);
+kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, float* x, cudaStream_t st);
+// out_bf16[r] / out_f32[r] = RMSNorm(x[idx ? idx[r] : r]) * g   (one of the outputs may be NULL)
+kvb_status launch_rmsnorm(const float* x, const int32_t* idx, int64_t m, int H, const float* g, float eps,
+                          uint16_t* out_bf16, float* out_f32, cudaStream_t st);
+kvb_status launch_gather_rows(const float* src, const int32_t* idx, int64_t m, int H, float* dst, cudaStream_t st);
+kvb_status launch_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const int32_t* dst_idx, int64_t m,
+                          int kv_dim, uint16_t* k_dst, uint16_t* v_dst, cudaStream_t st);
+kvb_status launch_iota(int32_t* out, int64_t n, int32_t start, cudaStream_t st);
+kvb_status launch_concat_rows(const int32_t* sel, int64_t k, int64_t n_ctx, int64_t n_query, int32_t* rows,
+                              cudaStream_t st);
+
+// ---------------------------------------------------------------- HKVD + top-k
+size_t hkvd_ws_bytes(int64_t n_ctx);
+kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t* k_cached, int64_t ld_cached,
+                       int64_t n_ctx, int kv_dim, int64_t k, int32_t* sel_out, float* dev_out, void* scratch,
+                       cudaStream_t st);
+
+// ---------------------------------------------------------------- workspace
+// Layout of a caller workspace for up to n rows.
+struct Workspace {
+    int* status;       // device status word (first 256 bytes)
+    float* x_all;      // [n][H] fp32 residual, all rows
+    float* x_sel;      // [n][H] fp32 residual, recomputed rows
+    uint16_t* a;       // [n][H] bf16 normalised rows (GEMM A operand)
+    uint16_t* q;       // [n][Hq D] bf16
+    uint16_t* attn;    // [n][Hq D] bf16
+    uint16_t* h;       // [n][F] bf16 SwiGLU output
+    uint16_t* k_fresh; // [n][Hkv D] bf16 check-layer keys
+    float* dev;        // [n] fp32 deviation
+    int32_t* rows;     // [n] recomputed row indices
+    int32_t* ident;    // [n] 0..n-1
+    int32_t* sel;      // [n] selected indices
+    void* topk;        // top-k scratch
+    size_t bytes;
+};
+size_t workspace_layout(const kvb_config* cfg, int64_t n, void* base, Workspace* w);
+
+}  // namespace kvb

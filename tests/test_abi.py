@@ -1,0 +1,99 @@
+"""The C-ABI library builds, loads and exports every symbol include/kvblend.h declares;
+host-only entry points and argument validation work without a GPU."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import llama
+from oracle.llama import Shape
+from paper_2609_09768_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def kvb():
+    from paper_2609_09768_gb300 import build, kvblend
+    build.build()
+    kvblend.lib()
+    return kvblend
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "kvblend.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvb_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(kvb):
+    names = header_functions()
+    assert len(names) >= 15
+    lib = C.CDLL(kvb.lib_path())
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(kvb.EXPORTED), set(names) ^ set(kvb.EXPORTED)
+
+
+def test_status_strings_and_version(kvb):
+    L = kvb.lib()
+    assert L.kvb_version() >= 100
+    for code, text in kvb.STATUS.items():
+        assert L.kvb_status_string(code).decode() == text
+
+
+def test_rope_table_matches_oracle(kvb):
+    for shape in (synth.TINY, synth.LLAMA8B):
+        cfg = kvb.config(shape)
+        cos, sin = kvb.rope_table_fill(cfg, 130000)
+        pos = np.array([0, 1, 2, 511, 8191, 8192, 65537, 124031, 129999])
+        c, s = llama.rope_cos_sin(Shape.of(shape), pos)
+        assert np.max(np.abs(cos[pos] - c)) < 1e-6 and np.max(np.abs(sin[pos] - s)) < 1e-6
+
+
+def test_workspace_size_grows_with_rows(kvb):
+    cfg = kvb.config(synth.LLAMA8B)
+    a, b = kvb.workspace_size(cfg, 1000), kvb.workspace_size(cfg, 124032)
+    assert 0 < a < b
+    # residuals (2 x fp32), bf16 activations and the MLP intermediate for 124k rows
+    assert b > 124032 * 4096 * (4 + 4 + 2) + 124032 * 14336 * 2
+
+
+def test_host_validation_rejects_bad_arguments(kvb):
+    L = kvb.lib()
+    cfg = kvb.config(synth.TINY)
+    # NULL config / pointers are rejected before any device work
+    assert L.kvb_rope_table_fill(None, 10, None, None) == kvb.KVB_ERR_INVALID_ARG
+    assert L.kvb_selective_prefill(None, None, None, None, None, None, None, None, 0, 0, 0, 0.15, 1, None, 0, None,
+                                   None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+    assert b"config is NULL" in L.kvb_last_error()
+    bad = kvb.config(synth.TINY)
+    bad.head_dim = 96
+    n = C.c_size_t(0)
+    assert L.kvb_workspace_size(C.byref(bad), 10, C.byref(n)) == kvb.KVB_ERR_UNSUPPORTED
+    bad = kvb.config(synth.TINY)
+    bad.n_kv_heads = 3
+    assert L.kvb_workspace_size(C.byref(bad), 10, C.byref(n)) == kvb.KVB_ERR_UNSUPPORTED
+    # k > n_ctx, misaligned leading dims
+    assert L.kvb_hkvd_select(None, 128, None, 128, 10, 128, 11, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+    assert L.kvb_hkvd_select(None, 12, None, 12, 10, 12, 1, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+    # misaligned pointer
+    assert L.kvb_kv_scatter(8, 16, 16, 1, 128, 16, 16, 4, None) == kvb.KVB_ERR_INVALID_ARG
+    assert b"aligned" in L.kvb_last_error()
+    # r outside [0, 1] and a check layer outside [1, L]
+    mw = kvb.ModelStruct()
+    assert L.kvb_selective_prefill(C.byref(cfg), C.byref(mw), None, None, None, None, None, None, 1, 10, 2, 1.5, 1,
+                                   None, 0, None, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+    # empty inputs are valid no-ops
+    assert L.kvb_kv_scatter(None, None, None, 0, 128, None, None, 4, None) == kvb.KVB_OK
+    assert L.kvb_hkvd_select(None, 128, None, 128, 0, 128, 0, None, None, None, 0, None) == kvb.KVB_OK
+
+
+def test_binding_fails_loudly_without_library(monkeypatch):
+    from paper_2609_09768_gb300 import kvblend
+    monkeypatch.setattr(kvblend, "_LIB", None)
+    monkeypatch.setattr(kvblend, "LIB", "/nonexistent/libkvblend.so")
+    with pytest.raises(RuntimeError, match="not built"):
+        kvblend.lib()

@@ -1,0 +1,217 @@
+"""Per-step parity of the CUDA path (through the C ABI) against the float64 oracle,
+on seeded synthetic inputs of both model shapes, with ragged sizes and edge cases."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import blend, llama
+from oracle.llama import Shape
+from paper_2609_09768_gb300 import synth
+from tests.gpu_util import (assert_close_abs, assert_close_rel, check_selection, errs, np64)
+
+pytestmark = pytest.mark.gpu
+
+TINY = synth.TINY
+L8B = synth.LLAMA8B.with_layers(2)
+
+
+@pytest.fixture(scope="module")
+def kvb():
+    from paper_2609_09768_gb300 import kvblend
+    kvblend.lib()
+    return kvblend
+
+
+def dev(t):
+    return t.to("cuda")
+
+
+# ------------------------------------------------------------------------------------------ realign
+
+@pytest.mark.parametrize("shape,starts", [
+    (TINY, [0, 128, 256, 384, 512]),
+    (L8B, synth.chunk_starts_equal(8, 480)),
+    (TINY, [0, 1, 70, 200, 203, 333]),            # ragged chunk lengths, a 1-token chunk
+])
+def test_realign_matches_oracle(kvb, shape, starts):
+    cfg = kvb.config(shape)
+    n_ctx, L, Hkv, D = starts[-1], shape.n_layers, shape.n_kv_heads, shape.head_dim
+    k_src = synth.randn_bf16((L, n_ctx, Hkv, D), 101)
+    v_src = synth.randn_bf16((L, n_ctx, Hkv, D), 102)
+    rope = kvb.RopeTable(cfg, n_ctx)
+    cs = dev(torch.tensor(starts, dtype=torch.int32))
+    rows = n_ctx + 13
+    k_dst = torch.zeros(L, rows, Hkv, D, dtype=torch.bfloat16, device="cuda")
+    v_dst = torch.zeros_like(k_dst)
+    kvb.rope_realign(cfg, rope, dev(k_src), dev(v_src), k_dst, v_dst, 0, L, cs, n_ctx)
+    torch.cuda.synchronize()
+    ref = blend.realign(Shape.of(shape), np64(k_src), starts)
+    e = assert_close_rel(k_dst[:, :n_ctx].cpu(), ref, "realigned K")
+    assert torch.equal(v_dst[:, :n_ctx].cpu(), v_src), "V must be copied bit-exactly"
+    assert torch.count_nonzero(k_dst[:, n_ctx:]) == 0, "rows past n_ctx must be untouched"
+    # in place gives the same bits as out of place
+    k_in = dev(k_src).clone()
+    kvb.rope_realign(cfg, rope, k_in, None, k_in, None, 0, L, cs, n_ctx)
+    torch.cuda.synchronize()
+    assert torch.equal(k_in, k_dst[:, :n_ctx])
+    print("realign", shape.head_dim, e)
+
+
+# ------------------------------------------------------------------------------------------ HKVD
+
+@pytest.mark.parametrize("n,kv_dim,k", [
+    (512, 128, 76), (3840, 1024, 576), (1000, 64, 333), (17, 128, 0), (17, 128, 17), (1, 128, 1),
+    (123904, 1024, 18585), (5000, 1024, 1),
+])
+def test_hkvd_select_matches_oracle(kvb, n, kv_dim, k):
+    kf = synth.randn_bf16((n, kv_dim), 201)
+    kc = synth.randn_bf16((n, kv_dim), 202)
+    # a band of rows with zero deviation (a prefix chunk) and duplicated rows (exact ties)
+    z = min(n // 4, 300)
+    kc[:z] = kf[:z]
+    if n > 40:
+        kf[20:30] = kf[10]
+        kc[20:30] = kc[10]
+    sel, dv = kvb.hkvd_select(dev(kf), dev(kc), k)
+    torch.cuda.synchronize()
+    dref = blend.hkvd_deviation(np64(kf), np64(kc))
+    e = errs(dv.cpu(), dref)
+    assert e["max_abs"] <= 1e-5 * max(1.0, float(dref.max())), e
+    s = sel.cpu().numpy()
+    assert np.all(np.diff(s) > 0), "indices must be ascending and distinct"
+    nd = check_selection(s, dref, k)
+    print("hkvd", n, k, "dev err", e["max_abs"], "differing (near-tie) indices", nd)
+
+
+def test_hkvd_exact_ties_take_lowest_index(kvb):
+    n, kv_dim = 4096, 256
+    kf = synth.randn_bf16((n, kv_dim), 203)
+    kc = kf.clone()
+    kc[:, 0] = kc[:, 0] + 1.0      # same-magnitude offsets on many rows -> many equal deviations
+    kc[::3, 1] = kc[::3, 1] + 2.0
+    for k in (1, 100, 1365, 1366, 2000, n):
+        sel, dv = kvb.hkvd_select(dev(kf), dev(kc), k)
+        d32 = dv.cpu().numpy()
+        want = blend.topk_select(d32.astype(np.float64), k)   # oracle rule on the GPU's own fp32 values
+        assert np.array_equal(sel.cpu().numpy(), want), k
+
+
+# ------------------------------------------------------------------------------------------ QKV GEMM
+
+@pytest.mark.parametrize("shape,m,n_src", [(TINY, 108, 544), (L8B, 640, 3904), (L8B, 1, 7), (TINY, 129, 300),
+                                           (L8B, 300, 300)])
+def test_gather_rmsnorm_qkv_matches_oracle(kvb, shape, m, n_src):
+    cfg = kvb.config(shape)
+    lw = synth.make_layer_weights(shape, 1, seed=5)
+    lwd = {k: dev(v) for k, v in lw.items()}
+    s = Shape.of(shape)
+    g = torch.Generator().manual_seed(7)
+    x = torch.randn(n_src, shape.hidden, generator=g) * 2.0
+    row_idx = torch.sort(torch.randperm(n_src, generator=g)[:m]).values.to(torch.int32)
+    max_pos = n_src + 50
+    rope_pos = torch.randint(0, max_pos, (m,), generator=g, dtype=torch.int32)
+    n_cache = n_src + 5
+    kv_dst = torch.randperm(n_cache, generator=g)[:m].to(torch.int32)
+    rope = kvb.RopeTable(cfg, max_pos)
+    q = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
+    kc = torch.zeros(n_cache, shape.kv_dim, dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros_like(kc)
+    ws = kvb.workspace(cfg, m)
+    kvb.gather_rmsnorm_qkv(cfg, kvb.layer_struct(lwd), rope, dev(x), dev(row_idx), dev(rope_pos), m, q, kc, vc,
+                           dev(kv_dst), ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    qr, kr, vr = llama.qkv_rows(s, lw, np64(x)[row_idx.numpy()], rope_pos.numpy())
+    eq = assert_close_rel(q.cpu(), qr.reshape(m, -1), "q")
+    ek = assert_close_rel(kc.cpu()[kv_dst.long()], kr.reshape(m, -1), "k")
+    ev = assert_close_rel(vc.cpu()[kv_dst.long()], vr.reshape(m, -1), "v")
+    untouched = torch.ones(n_cache, dtype=torch.bool)
+    untouched[kv_dst.long()] = False
+    assert torch.count_nonzero(kc.cpu()[untouched]) == 0
+    print("qkv", shape.hidden, m, eq, ek, ev)
+
+
+# ------------------------------------------------------------------------------------------ attention
+
+def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
+    cfg = kvb.config(shape)
+    m = len(q_rows)
+    q = synth.randn_bf16((m, shape.n_q_heads, shape.head_dim), seed)
+    k = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 1)
+    v = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 2)
+    qi = torch.tensor(q_rows, dtype=torch.int32)
+    lo = None if kv_lo is None else torch.tensor(kv_lo, dtype=torch.int32)
+    out = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    kvb.sparse_query_attn(cfg, dev(q), dev(qi), None if lo is None else dev(lo), dev(k), dev(v), out, ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    ref = llama.attention_rows(Shape.of(shape), np64(q), np64(k), np64(v), q_rows, kv_lo)
+    return out.cpu(), ref.reshape(m, -1)
+
+
+@pytest.mark.parametrize("shape,n_kv", [(TINY, 544), (L8B, 3904), (TINY, 1), (L8B, 130), (L8B, 129)])
+def test_attention_dense_causal(kvb, shape, n_kv):
+    out, ref = _attn_case(kvb, shape, n_kv, list(range(n_kv)))
+    e = assert_close_rel(out, ref, "dense causal attention")
+    print("attn dense", shape.head_dim, n_kv, e)
+
+
+@pytest.mark.parametrize("shape,n_kv,m", [(TINY, 544, 108), (L8B, 3904, 640), (L8B, 3904, 33), (L8B, 5000, 1),
+                                          (TINY, 200, 3)])
+def test_attention_sparse_rows(kvb, shape, n_kv, m):
+    g = np.random.default_rng(m)
+    rows = np.sort(g.choice(n_kv, size=m, replace=False))
+    rows[-1] = n_kv - 1
+    out, ref = _attn_case(kvb, shape, n_kv, rows.tolist())
+    e = assert_close_rel(out, ref, "sparse-query attention")
+    print("attn sparse", shape.head_dim, n_kv, m, e)
+
+
+@pytest.mark.parametrize("shape,starts", [(TINY, [0, 128, 256, 384, 512]), (L8B, [0, 480, 960, 1440]),
+                                          (TINY, [0, 5, 140, 141, 300])])
+def test_attention_block_diagonal(kvb, shape, starts):
+    n = starts[-1]
+    lo = np.concatenate([[starts[c]] * (starts[c + 1] - starts[c]) for c in range(len(starts) - 1)])
+    out, ref = _attn_case(kvb, shape, n, list(range(n)), lo.tolist())
+    e = assert_close_rel(out, ref, "block-diagonal attention")
+    print("attn blockdiag", shape.head_dim, e)
+
+
+# ------------------------------------------------------------------------------------------ MLP half
+
+@pytest.mark.parametrize("shape,m", [(TINY, 108), (L8B, 640), (L8B, 1), (TINY, 300)])
+def test_mlp_rows_matches_oracle(kvb, shape, m):
+    cfg = kvb.config(shape)
+    lw = synth.make_layer_weights(shape, 0, seed=9)
+    lwd = {k: dev(v) for k, v in lw.items()}
+    attn = synth.randn_bf16((m, shape.q_dim), 301)
+    g = torch.Generator().manual_seed(3)
+    x = torch.randn(m, shape.hidden, generator=g) * 1.5
+    xd = dev(x).contiguous()
+    ws = kvb.workspace(cfg, m)
+    kvb.mlp_rows(cfg, kvb.layer_struct(lwd), dev(attn), xd, ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    ref = llama.attn_out_mlp(Shape.of(shape), lw, np64(x), np64(attn))
+    e = assert_close_abs(xd.cpu(), ref, "x after O-proj + MLP")
+    print("mlp", shape.hidden, m, e)
+
+
+# ------------------------------------------------------------------------------------------ scatter
+
+@pytest.mark.parametrize("m,kv_dim,n_dst", [(576, 1024, 3904), (1, 128, 5), (108, 128, 544), (0, 128, 4)])
+def test_kv_scatter_bit_exact(kvb, m, kv_dim, n_dst):
+    g = torch.Generator().manual_seed(m)
+    kr = synth.randn_bf16((m, kv_dim), 401)
+    vr = synth.randn_bf16((m, kv_dim), 402)
+    idx = torch.randperm(n_dst, generator=g)[:m].to(torch.int32)
+    kd = torch.zeros(n_dst, kv_dim, dtype=torch.bfloat16, device="cuda")
+    vd = torch.zeros_like(kd)
+    kvb.kv_scatter(dev(kr), dev(vr), dev(idx), kd, vd)
+    torch.cuda.synchronize()
+    want_k = torch.zeros(n_dst, kv_dim, dtype=torch.bfloat16)
+    want_v = torch.zeros_like(want_k)
+    want_k[idx.long()] = kr
+    want_v[idx.long()] = vr
+    assert torch.equal(kd.cpu(), want_k) and torch.equal(vd.cpu(), want_v)
