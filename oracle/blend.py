@@ -35,7 +35,7 @@ from typing import Optional, Sequence
 
 import numpy as np
 
-from .llama import (F64, Shape, as64, apply_rope, attn_out_mlp, k_rows, layer_rows,
+from .llama import (F64, Shape, act, as64, apply_rope, attn_out_mlp, k_rows, layer_rows,
                     rmsnorm, rope_cos_sin)
 
 
@@ -104,7 +104,7 @@ def realign(s: Shape, k_local: np.ndarray, chunk_starts: Sequence[int]) -> np.nd
         rot = apply_rope(flat, np.broadcast_to(cos, (flat.shape[0], cos.shape[1])),
                          np.broadcast_to(sin, (flat.shape[0], sin.shape[1])))
         k[..., a:b, :, :] = rot.reshape(shp)
-    return k
+    return act(s, k)
 
 
 def hkvd_deviation(k_fresh, k_cached) -> np.ndarray:

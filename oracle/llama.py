@@ -16,6 +16,14 @@ the selective recompute of Sec. 3.2 (selected rows over the whole blended cache)
 RoPE is the rotate-half form used by Llama: dimension i is paired with i + D/2
 and the pair is rotated by angle pos * w_i, w_i = theta^(-2i/D), with Llama 3.1's
 frequency scaling (factor, low/high frequency factors, original context).
+
+Precision.  Arithmetic is float64.  Sec. 4 of the paper states that the model's
+computations run in bfloat16 (only the position adjustment in float32).  With
+`Shape.act_bf16` set, the oracle stores in bf16 exactly the activations such a
+model holds in bf16 - the RMSNorm outputs that feed a linear layer, q/k/v after
+RoPE (k and v are the KV cache), the attention output, the SwiGLU product and
+the re-aligned cached keys - and keeps everything else (accumulation, softmax,
+the residual stream) in float64.  Without it every tensor stays float64.
 """
 from __future__ import annotations
 
@@ -42,13 +50,14 @@ class Shape:
     rs_low: float = 1.0
     rs_high: float = 4.0
     rs_orig_ctx: int = 8192
+    act_bf16: bool = False
 
     @staticmethod
-    def of(s) -> "Shape":
+    def of(s, act_bf16: bool = False) -> "Shape":
         """Copy the fields from any object that has them (e.g. a ModelShape)."""
         return Shape(s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.mlp_dim,
                      float(s.rms_eps), float(s.rope_theta), bool(s.rope_llama3),
-                     float(s.rs_factor), float(s.rs_low), float(s.rs_high), int(s.rs_orig_ctx))
+                     float(s.rs_factor), float(s.rs_low), float(s.rs_high), int(s.rs_orig_ctx), act_bf16)
 
 
 def as64(a) -> np.ndarray:
@@ -59,6 +68,18 @@ def as64(a) -> np.ndarray:
             a = a.float()
         a = a.numpy()
     return np.asarray(a, dtype=F64)
+
+
+def bf16_round(x) -> np.ndarray:
+    """Round to the nearest bfloat16 (ties to even) through torch's conversion, as float64."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32))
+    return t.to(torch.bfloat16).to(torch.float64).numpy()
+
+
+def act(s: "Shape", x: np.ndarray) -> np.ndarray:
+    """An activation the model stores: bf16 when s.act_bf16, else unchanged."""
+    return bf16_round(x) if s.act_bf16 else x
 
 
 # ----------------------------------------------------------------------------- RoPE
@@ -171,31 +192,31 @@ def attention_rows(s: Shape, q: np.ndarray, k_cache: np.ndarray, v_cache: np.nda
 def qkv_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> tuple[np.ndarray, np.ndarray, np.ndarray]:
     """RMSNorm -> QKV projection -> RoPE at `rope_pos`.  Returns q [m,Hq,D], k, v [m,Hkv,D]."""
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
-    n1 = rmsnorm(x, lw["attn_norm"], s.rms_eps)
+    n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
     qkv = linear(n1, lw["w_qkv"])
     m = x.shape[0]
     q = qkv[:, : Hq * D].reshape(m, Hq, D)
     k = qkv[:, Hq * D: (Hq + Hkv) * D].reshape(m, Hkv, D)
     v = qkv[:, (Hq + Hkv) * D:].reshape(m, Hkv, D)
     c, sn = rope_cos_sin(s, rope_pos)
-    return apply_rope(q, c, sn), apply_rope(k, c, sn), v
+    return act(s, apply_rope(q, c, sn)), act(s, apply_rope(k, c, sn)), act(s, v)
 
 
 def k_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> np.ndarray:
     """Only the key projection (RMSNorm -> W_k -> RoPE), [m, Hkv, D]."""
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
-    n1 = rmsnorm(x, lw["attn_norm"], s.rms_eps)
+    n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
     wk = as64(lw["w_qkv"])[Hq * D: (Hq + Hkv) * D]
     k = (n1 @ wk.T).reshape(x.shape[0], Hkv, D)
     c, sn = rope_cos_sin(s, rope_pos)
-    return apply_rope(k, c, sn)
+    return act(s, apply_rope(k, c, sn))
 
 
 def attn_out_mlp(s: Shape, lw: dict, x: np.ndarray, attn: np.ndarray) -> np.ndarray:
     """x + O-proj(attn), then + SwiGLU MLP of its RMSNorm.  attn: [m, Hq*D]."""
     h = as64(x) + linear(attn, lw["w_o"])
-    n2 = rmsnorm(h, lw["mlp_norm"], s.rms_eps)
-    a = silu(linear(n2, lw["w_gate"])) * linear(n2, lw["w_up"])
+    n2 = act(s, rmsnorm(h, lw["mlp_norm"], s.rms_eps))
+    a = act(s, silu(linear(n2, lw["w_gate"])) * linear(n2, lw["w_up"]))
     return h + linear(a, lw["w_down"])
 
 
@@ -211,5 +232,5 @@ def layer_rows(s: Shape, lw: dict, x: np.ndarray, row_idx, rope_pos, k_cache: np
     q, k, v = qkv_rows(s, lw, x, rope_pos)
     k_cache[row_idx] = k
     v_cache[row_idx] = v
-    a = attention_rows(s, q, k_cache, v_cache, row_idx, row_lo)
+    a = act(s, attention_rows(s, q, k_cache, v_cache, row_idx, row_lo))
     return attn_out_mlp(s, lw, x, a.reshape(a.shape[0], -1))

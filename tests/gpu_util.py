@@ -4,15 +4,32 @@ Tolerances (float outputs are compared with the float64 oracle on the same
 bf16-representable inputs):
   * layer outputs / final hidden states: max-abs <= 2e-2 and mean-abs <= 2e-3
     (the bar the method's specification states for bf16 outputs);
-  * bf16 intermediates (q, k, v, attention output, realigned keys): errors are
-    judged relative to the reference RMS, max <= 2e-2 * rms and mean <= 2e-3 * rms,
-    i.e. the same bar applied to a unit-scale signal.  One bf16 rounding of the
-    result alone contributes up to 2^-9 (0.2 %) relative per element.
+  * bf16 intermediates (q, k, v, realigned keys): errors are judged relative to
+    the reference RMS, max <= 2e-2 * rms and mean <= 2e-3 * rms, i.e. the same bar
+    applied to a unit-scale signal.  One bf16 rounding of the result alone
+    contributes up to 2^-9 (0.2 %) relative per element.
+  * attention outputs: the same bar relative to the RMS of V.  The output is a
+    convex combination of value rows; rounding each softmax weight to bf16 (the
+    P operand of the P.V product) perturbs it by at most 2^-9 * max|v - out|,
+    which scales with the values, not with the (much smaller) RMS of the average.
 """
 import numpy as np
 import torch
 
 MAX_ABS, MEAN_ABS = 2e-2, 2e-3
+
+
+def fp64_gap_bounds(rms: float, n_layers: int) -> tuple:
+    """Bound on the gap between the GPU path and the all-float64 oracle.
+
+    The CUDA path holds five activations per layer in bf16 (the oracle's act_bf16
+    mode rounds the same ones); each rounding is at most 2^-9 relative, RMS
+    2^-9/sqrt(3), and the layer maps carry it into the residual with gain ~1, so
+    the RMS gap after L layers is about 2^-9 * sqrt(5 L / 3) of the signal.  We
+    allow mean-abs <= 2^-9 * sqrt(5 L) * rms and max-abs <= 8x that.
+    """
+    mean = 2.0 ** -9 * np.sqrt(5.0 * n_layers) * rms
+    return 8.0 * mean, mean
 
 
 def np64(t) -> np.ndarray:
@@ -40,10 +57,10 @@ def assert_close_abs(got, want, what="", max_abs=MAX_ABS, mean_abs=MEAN_ABS):
     return e
 
 
-def assert_close_rel(got, want, what="", max_rel=MAX_ABS, mean_rel=MEAN_ABS):
+def assert_close_rel(got, want, what="", max_rel=MAX_ABS, mean_rel=MEAN_ABS, scale=None):
     e = errs(got, want)
     assert np.all(np.isfinite(np64(got))), f"{what}: non-finite values"
-    s = max(e["rms_ref"], 1e-30)
+    s = max(e["rms_ref"] if scale is None else scale, 1e-30)
     assert e["max_abs"] <= max_rel * s and e["mean_abs"] <= mean_rel * s, f"{what}: {e}"
     return e
 

@@ -45,7 +45,7 @@ def test_realign_matches_oracle(kvb, shape, starts):
     v_dst = torch.zeros_like(k_dst)
     kvb.rope_realign(cfg, rope, dev(k_src), dev(v_src), k_dst, v_dst, 0, L, cs, n_ctx)
     torch.cuda.synchronize()
-    ref = blend.realign(Shape.of(shape), np64(k_src), starts)
+    ref = blend.realign(Shape.of(shape, act_bf16=True), np64(k_src), starts)
     e = assert_close_rel(k_dst[:, :n_ctx].cpu(), ref, "realigned K")
     assert torch.equal(v_dst[:, :n_ctx].cpu(), v_src), "V must be copied bit-exactly"
     assert torch.count_nonzero(k_dst[:, n_ctx:]) == 0, "rows past n_ctx must be untouched"
@@ -104,7 +104,7 @@ def test_gather_rmsnorm_qkv_matches_oracle(kvb, shape, m, n_src):
     cfg = kvb.config(shape)
     lw = synth.make_layer_weights(shape, 1, seed=5)
     lwd = {k: dev(v) for k, v in lw.items()}
-    s = Shape.of(shape)
+    s = Shape.of(shape, act_bf16=True)
     g = torch.Generator().manual_seed(7)
     x = torch.randn(n_src, shape.hidden, generator=g) * 2.0
     row_idx = torch.sort(torch.randperm(n_src, generator=g)[:m]).values.to(torch.int32)
@@ -147,13 +147,13 @@ def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
     torch.cuda.synchronize()
     assert kvb.device_status(ws) == 0
     ref = llama.attention_rows(Shape.of(shape), np64(q), np64(k), np64(v), q_rows, kv_lo)
-    return out.cpu(), ref.reshape(m, -1)
+    return out.cpu(), ref.reshape(m, -1), float(np.sqrt(np.mean(np64(v) ** 2)))
 
 
 @pytest.mark.parametrize("shape,n_kv", [(TINY, 544), (L8B, 3904), (TINY, 1), (L8B, 130), (L8B, 129)])
 def test_attention_dense_causal(kvb, shape, n_kv):
-    out, ref = _attn_case(kvb, shape, n_kv, list(range(n_kv)))
-    e = assert_close_rel(out, ref, "dense causal attention")
+    out, ref, vs = _attn_case(kvb, shape, n_kv, list(range(n_kv)))
+    e = assert_close_rel(out, ref, "dense causal attention", scale=vs)
     print("attn dense", shape.head_dim, n_kv, e)
 
 
@@ -163,8 +163,8 @@ def test_attention_sparse_rows(kvb, shape, n_kv, m):
     g = np.random.default_rng(m)
     rows = np.sort(g.choice(n_kv, size=m, replace=False))
     rows[-1] = n_kv - 1
-    out, ref = _attn_case(kvb, shape, n_kv, rows.tolist())
-    e = assert_close_rel(out, ref, "sparse-query attention")
+    out, ref, vs = _attn_case(kvb, shape, n_kv, rows.tolist())
+    e = assert_close_rel(out, ref, "sparse-query attention", scale=vs)
     print("attn sparse", shape.head_dim, n_kv, m, e)
 
 
@@ -173,8 +173,8 @@ def test_attention_sparse_rows(kvb, shape, n_kv, m):
 def test_attention_block_diagonal(kvb, shape, starts):
     n = starts[-1]
     lo = np.concatenate([[starts[c]] * (starts[c + 1] - starts[c]) for c in range(len(starts) - 1)])
-    out, ref = _attn_case(kvb, shape, n, list(range(n)), lo.tolist())
-    e = assert_close_rel(out, ref, "block-diagonal attention")
+    out, ref, vs = _attn_case(kvb, shape, n, list(range(n)), lo.tolist())
+    e = assert_close_rel(out, ref, "block-diagonal attention", scale=vs)
     print("attn blockdiag", shape.head_dim, e)
 
 
@@ -193,7 +193,7 @@ def test_mlp_rows_matches_oracle(kvb, shape, m):
     kvb.mlp_rows(cfg, kvb.layer_struct(lwd), dev(attn), xd, ws)
     torch.cuda.synchronize()
     assert kvb.device_status(ws) == 0
-    ref = llama.attn_out_mlp(Shape.of(shape), lw, np64(x), np64(attn))
+    ref = llama.attn_out_mlp(Shape.of(shape, act_bf16=True), lw, np64(x), np64(attn))
     e = assert_close_abs(xd.cpu(), ref, "x after O-proj + MLP")
     print("mlp", shape.hidden, m, e)
 

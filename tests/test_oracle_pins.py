@@ -387,3 +387,40 @@ def test_planted_mistakes(monkeypatch):
     def freq_bad(s):                   # exponent -i/D instead of -2i/D
         return good_freq(s) ** 0.5
     assert _pins_fail(monkeypatch, llama, "rope_inv_freq", freq_bad)
+
+
+# ------------------------------------------------------------------------------------ bf16 storage mode
+
+def test_bf16_round_is_round_to_nearest_even():
+    """Against the bit-level definition: keep the top 16 bits of the fp32 pattern,
+    rounding the dropped 16 bits to nearest with ties to an even kept part."""
+    rng = np.random.default_rng(11)
+    x = np.concatenate([rng.standard_normal(5000) * 10.0 ** rng.integers(-6, 6, 5000),
+                        [1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -1.0 - 2.0 ** -8, 0.0, 65504.0]]).astype(np.float32)
+    b = x.view(np.uint32).astype(np.uint64)
+    r = ((b + 0x7FFF + ((b >> 16) & 1)) >> 16) << 16
+    want = r.astype(np.uint32).view(np.float32).astype(np.float64)
+    assert np.array_equal(llama.bf16_round(x), want)
+    assert llama.bf16_round([1.0 + 2.0 ** -8])[0] == 1.0            # tie -> even
+    assert llama.bf16_round([1.0 + 3 * 2.0 ** -8])[0] == 1.0 + 2.0 ** -6
+
+
+def test_bf16_storage_mode_rounds_only_stored_activations():
+    """With act_bf16 the cache entries are bf16 values, the residual stream is not, and the
+    result stays within bf16 rounding of the float64 one; without it nothing is rounded."""
+    shape = MINI.with_layers(2)
+    m = model(shape)
+    starts = [0, 9, 20]
+    toks = synth.make_tokens(shape, 25, 1)
+    x0 = blend.embed_rows(m["embed"], toks.numpy())
+    s16, s64 = Shape.of(shape, act_bf16=True), Shape.of(shape)
+    r16 = blend.full_prefill(s16, m["layers_np"], x0)
+    r64 = blend.full_prefill(s64, m["layers_np"], x0)
+    assert np.array_equal(llama.bf16_round(r16["k"]), r16["k"]) and np.array_equal(llama.bf16_round(r16["v"]), r16["v"])
+    assert not np.array_equal(llama.bf16_round(r16["x"]), r16["x"])
+    assert not np.array_equal(llama.bf16_round(r64["k"]), r64["k"])
+    g = rel(r16["x"], r64["x"])
+    assert 1e-5 < g < 2e-2
+    cc = blend.chunk_caches(s16, m["layers_np"], x0[:20], starts)
+    re = blend.realign(s16, cc["k"], starts)
+    assert np.array_equal(llama.bf16_round(re), re)
