@@ -1,0 +1,372 @@
+#!/usr/bin/env python
+"""Benchmark: time to first token of the selective-recompute prefill on one GB300.
+
+A step is one call of kvb_selective_prefill on the headline workload: a 32-layer
+Llama-3.1-8B-shaped bf16 model (random weights), 242 chunks x 512 tokens of
+per-chunk KV caches resident in HBM plus a 128-token query (124,032 tokens),
+recompute ratio r = 0.15.  The step covers merge + re-alignment of the chunk
+caches, the dense layer 0, the HKVD selection and the 31 selective layers, up
+to the query rows' final hidden state.  `value` is the mean TTFT in ms over the
+timed steps (lower is better).  Next to it the line reports the library's own
+dense r = 1.0 prefill of the same request, the end-to-end TTFT with the chunk
+caches copied from pinned host memory inside the timed region, a live roofline
+of the dominant kernel and the CPU oracle's time on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With --gpus N under torchrun every rank serves its own replica of the request
+(no data-path collective; the path has no exchange step).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % of bf16 peak"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="l8b_124k")
+    ap.add_argument("--r", type=float, default=None)
+    ap.add_argument("--r1-steps", type=int, default=1, help="timed steps of the r = 1.0 comparator (0: skip)")
+    ap.add_argument("--e2e-steps", type=int, default=2, help="timed end-to-end steps (0: skip)")
+    ap.add_argument("--cpu-rows", type=int, default=512, help="rows in the oracle's timed sample")
+    ap.add_argument("--no-cpu", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16": p["bf16_tflops"], "bf16_sustained": p["bf16_tflops_sustained"],
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+class Clocks:
+    """nvidia-smi sampling (200 ms) while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.rows, self.proc = index, [], None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([c.strip() for c in line.split(",")])
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        time.sleep(0.1)
+        sm = [float(r[1]) for r in self.rows if len(r) >= 9 and r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in self.rows if len(r) >= 9 and r[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in self.rows:
+            if len(r) >= 9:
+                for n, v in zip(names, r[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------ oracle (CPU) leg
+
+class OracleSample:
+    """A bounded sample of the workload for the CPU oracle: one selective decoder layer
+    over `n_rows` rows spread uniformly over the context, attending a float64 cache of
+    the full request length.  Inputs are drawn once; run() times the oracle call."""
+
+    def __init__(self, wl, n_rows: int, seed: int = 0):
+        import numpy as np
+        from oracle import llama
+        from oracle.llama import Shape
+        from paper_2609_09768_gb300 import synth
+        shape = wl.shape
+        self.s = Shape.of(shape, act_bf16=True)
+        self.lw = {k: llama.as64(v) for k, v in synth.make_layer_weights(shape, 1, seed).items()}
+        N = wl.n_total
+        rng = np.random.default_rng(seed)
+        self.kc = rng.standard_normal((N, shape.n_kv_heads, shape.head_dim))
+        self.vc = rng.standard_normal((N, shape.n_kv_heads, shape.head_dim))
+        self.rows = np.sort(rng.choice(wl.n_ctx, size=n_rows, replace=False))
+        self.x = rng.standard_normal((n_rows, shape.hidden))
+        self.n_rows = n_rows
+
+    def run(self) -> float:
+        from oracle import llama
+        t0 = time.perf_counter()
+        llama.layer_rows(self.s, self.lw, self.x, self.rows, self.rows, self.kc, self.vc)
+        return time.perf_counter() - t0
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_ttft_ms(wl, seconds: float, rows: int, k: int) -> float:
+    """Scale a sample to the prefill: layer 0 over all N rows plus (L-1) layers over m rows."""
+    m = k + wl.n_query
+    row_layers = wl.n_total + (wl.shape.n_layers - 1) * m
+    return seconds / rows * row_layers * 1e3
+
+
+def run_reference(args, wl, rank: int, world: int) -> None:
+    """The reference arm: the CPU oracle as it stands, on the host cores."""
+    if rank != 0:
+        return
+    from oracle import blend
+    r = wl.r if args.r is None else args.r
+    k = blend.num_selected(r, wl.n_ctx)
+    rows = max(16, min(64, args.cpu_rows))
+    smp = OracleSample(wl, rows)
+    for _ in range(args.warmup):
+        smp.run()
+    vals = []
+    for _ in range(args.steps):
+        vals.append(oracle_ttft_ms(wl, smp.run(), rows, k))
+    v = statistics.mean(vals)
+    sample = (f"oracle selective layer on {rows} of {k + wl.n_query} recomputed rows (uniform over the context) "
+              f"attending a {wl.n_total}-row cache, per step; scaled by (N + (L-1) m) row-layers")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "ms", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(v, 3), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "n_ctx": wl.n_ctx, "n_query": wl.n_query, "r": r, "k": k},
+        "cpu_baseline": {"value": round(v, 3), "unit": "ms", "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(v, 3), "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ------------------------------------------------------------------------------------ our arm
+
+def run_ours(args, wl, rank: int, world: int) -> None:
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2609_09768_gb300 import build, synth, workload
+    from paper_2609_09768_gb300 import kvblend as kvb
+
+    build.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    shape = wl.shape
+    r = wl.r if args.r is None else args.r
+    cfg = kvb.config(shape)
+    N, n_ctx, nq, L = wl.n_total, wl.n_ctx, wl.n_query, shape.n_layers
+    Hq, Hkv, D, H, F = shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.hidden, shape.mlp_dim
+    pk = peaks()
+
+    weights = workload.device_model(shape, seed=0, device=dev, draw_on_device=True)
+    model = kvb.Model(weights)
+    toks = synth.make_tokens(shape, N, 1).to(dev)
+    rope = kvb.RopeTable(cfg, N, dev)
+    ws = kvb.workspace(cfg, N, dev)
+    starts = wl.chunk_starts()
+    dstarts = torch.tensor(starts, dtype=torch.int32, device=dev)
+    kch, vch = workload.chunk_caches(cfg, model, rope, toks[:n_ctx], starts, ws=ws)
+    ck = torch.empty(L, N, Hkv, D, dtype=torch.bfloat16, device=dev)
+    cv = torch.empty_like(ck)
+    fh = torch.empty(nq, H, dtype=torch.float32, device=dev)
+    sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize()
+
+    def step(rr=r, timings=True):
+        return kvb.selective_prefill(cfg, model, rope, kch, vch, ck, cv, toks, dstarts, n_ctx, nq, rr, 1,
+                                     final_hidden=fh, sel_out=sel, ws=ws, timings=timings)[2]
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    clocks = Clocks(torch.cuda.current_device())
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    tims = [step() for _ in range(args.steps)]
+    e1.record()
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    assert kvb.device_status(ws) == 0, "device wait timed out"
+
+    # algorithmic work of the step (from the chosen rows, read back after the timed region)
+    k = int(tims[-1]["n_selected"])
+    m = k + nq
+    rows = np.concatenate([sel[:k].cpu().numpy().astype(np.int64), np.arange(n_ctx, N)])
+    attn_sel_flop = 4.0 * Hq * D * float(np.sum(rows + 1))          # per selective layer
+    attn_dense_flop = 4.0 * Hq * D * N * (N + 1) / 2.0               # layer 0
+    gemm_row_flop = 2.0 * H * (shape.qkv_dim + shape.q_dim) + 2.0 * 3 * H * F
+    gemm_flop = gemm_row_flop * (N + (L - 1) * m) + 2.0 * n_ctx * H * shape.kv_dim
+    total_flop = attn_dense_flop + (L - 1) * attn_sel_flop + gemm_flop
+
+    def avg(key):
+        return statistics.mean(t[key] for t in tims)
+
+    kern = {
+        "attn_selective": {"ms": avg("attn_sel_ms"), "launches": int(tims[-1]["n_attn_sel"]),
+                           "flop": attn_sel_flop * (L - 1)},
+        "attn_dense": {"ms": avg("attn_dense_ms"), "launches": int(tims[-1]["n_attn_dense"]), "flop": attn_dense_flop},
+        "gemm": {"ms": avg("gemm_ms"), "launches": int(tims[-1]["n_gemm"]), "flop": gemm_flop},
+    }
+    for v in kern.values():
+        v["tflops"] = v["flop"] / (v["ms"] * 1e-3) / 1e12 if v["ms"] > 0 else None
+        v["frac_of_sustained_peak"] = (v["tflops"] / pk["bf16_sustained"]) if v["tflops"] else None
+    dom_name = max(kern, key=lambda n: kern[n]["ms"])
+    dom = kern[dom_name]
+    per_launch_ms = dom["ms"] / max(dom["launches"], 1)
+    per_launch_flop = dom["flop"] / max(dom["launches"], 1)
+    achieved = per_launch_flop / (per_launch_ms * 1e-3) / 1e12
+    roofline = {"kernel": dom_name, "bound": "tensor", "achieved": round(achieved, 2),
+                "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": round(achieved / pk["bf16_sustained"], 4),
+                "traffic": None, "peak_source": f"{pk['source']} bf16 sustained",
+                "flop_per_launch": per_launch_flop, "ms_per_launch": round(per_launch_ms, 4)}
+
+    # the library's own dense r = 1.0 prefill of the same request
+    r1 = None
+    if args.r1_steps > 0:
+        step(1.0)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        r1t = [step(1.0) for _ in range(args.r1_steps)]
+        b.record()
+        torch.cuda.synchronize()
+        r1_ms = a.elapsed_time(b) / args.r1_steps
+        r1 = {"ttft_ms": round(r1_ms, 3), "attn_dense_ms": round(statistics.mean(t["attn_dense_ms"] for t in r1t), 3),
+              "gemm_ms": round(statistics.mean(t["gemm_ms"] for t in r1t), 3),
+              "attn_tflops": round(4.0 * Hq * D * N * (N + 1) / 2.0 * L /
+                                   (statistics.mean(t["attn_dense_ms"] for t in r1t) * 1e-3) / 1e12, 2)}
+
+    # end to end: chunk caches + tokens from pinned host memory, final hidden back to the host
+    e2e = None
+    if args.e2e_steps > 0:
+        hk = torch.empty(kch.shape, dtype=kch.dtype, pin_memory=True)
+        hv = torch.empty(vch.shape, dtype=vch.dtype, pin_memory=True)
+        ht = torch.empty(toks.shape, dtype=toks.dtype, pin_memory=True)
+        hf = torch.empty(fh.shape, dtype=fh.dtype, pin_memory=True)
+        hk.copy_(kch); hv.copy_(vch); ht.copy_(toks)
+        kd, vd, td = torch.empty_like(kch), torch.empty_like(vch), torch.empty_like(toks)
+        torch.cuda.synchronize()
+
+        def e2e_step():
+            kd.copy_(hk, non_blocking=True); vd.copy_(hv, non_blocking=True); td.copy_(ht, non_blocking=True)
+            kvb.selective_prefill(cfg, model, rope, kd, vd, ck, cv, td, dstarts, n_ctx, nq, r, 1,
+                                  final_hidden=fh, sel_out=sel, ws=ws)
+            hf.copy_(fh, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        b.record()
+        torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b) / args.e2e_steps
+        h2d = hk.numel() * 2 + hv.numel() * 2 + ht.numel() * 4
+        e2e = {"value": round(e2e_ms, 3), "unit": "ms", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(hf.numel() * 4)}
+        del hk, hv, kd, vd
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        n = args.cpu_rows
+        sec = OracleSample(wl, n).run()
+        cpu = {"value": round(oracle_ttft_ms(wl, sec, n, k), 1), "unit": "ms", "cores": cpu_cores(), "kind": "oracle",
+               "sample": (f"oracle selective layer on {n} of {m} recomputed rows (uniform over the context) "
+                          f"attending a {N}-row float64 cache, {sec:.1f} s; scaled by (N + (L-1) m) row-layers "
+                          f"(extrapolated)")}
+
+    if rank == 0:
+        stages = {k_: round(avg(k_), 3) for k_ in ("realign_ms", "dense_ms", "select_ms", "selective_ms", "final_ms")}
+        kdict = {n: {kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in v.items()}
+                 for n, v in kern.items()}
+        out = {
+            "metric": METRIC, "value": round(ms, 3), "unit": "ms", "n_gpus": world, "steps": args.steps,
+            "warmup": max(args.warmup, 3), "ms_per_step": round(ms, 3), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (random N(0,0.02) weights, uniform token ids, per-chunk caches from isolated prefill)",
+            "config": {"workload": wl.name, "n_layers": L, "n_chunks": wl.n_chunks, "chunk_len": wl.chunk_len,
+                       "n_ctx": n_ctx, "n_query": nq, "n_tokens": N, "r": r, "k": k, "check_layer": 1,
+                       "l2": "inputs larger than L2 (16.3 GB of chunk KV caches read per step)",
+                       "parallelism": f"replicas x{world}"},
+            "tokens_per_s": round(world * N / (ms * 1e-3), 1),
+            "r1_dense": r1,
+            "ttft_reduction_vs_r1": (round(1.0 - ms / r1["ttft_ms"], 4) if r1 else None),
+            "algorithmic_tflops": round(total_flop / (ms * 1e-3) / 1e12, 2),
+            "stages_ms": stages, "kernels": kdict,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": int(sum(t["n_launches"] for t in tims)),
+            "clocks": clk,
+        }
+        print(json.dumps(out))
+
+
+def main():
+    args = parse()
+    from paper_2609_09768_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+        return
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    run_ours(args, wl, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -104,7 +104,8 @@ typedef struct kvb_kv_cache {
     int32_t n_layers;
 } kvb_kv_cache;
 
-/* Stage times of one prefill in milliseconds (CUDA events on the call's stream). */
+/* Stage and kernel times of one prefill in milliseconds (CUDA events on the call's
+ * stream; kernel times are sums of per-launch event pairs). */
 typedef struct kvb_timings {
     float total_ms;
     float realign_ms;     /* merge + position re-alignment of the chunk caches      */
@@ -112,6 +113,11 @@ typedef struct kvb_timings {
     float select_ms;      /* check-layer keys, deviation and top-k                    */
     float selective_ms;   /* selective layers over the recomputed rows                */
     float final_ms;       /* final RMSNorm of the query rows                          */
+    float attn_dense_ms;  /* attention launches of the dense layers                  */
+    float attn_sel_ms;    /* attention launches of the selective layers              */
+    float gemm_ms;        /* all GEMM launches                                        */
+    int32_t n_attn_dense, n_attn_sel, n_gemm;
+    int32_t n_launches;   /* kernels this call launched                              */
     int64_t n_selected;   /* k = number of recomputed context rows                   */
     int64_t n_rows;       /* m = k + n_query                                          */
 } kvb_timings;

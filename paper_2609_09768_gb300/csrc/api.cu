@@ -7,8 +7,10 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "internal.h"
 
@@ -42,6 +44,10 @@ int num_sms() {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+static std::atomic<int64_t> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+int64_t launch_count() { return g_launches.load(std::memory_order_relaxed); }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -193,13 +199,54 @@ static void inv_freq(const kvb_config* c, double* w) {
 
 namespace {
 
+// Per-launch CUDA event pairs around the tensor-core kernels (only when timings are asked for).
+enum ProfKind { PK_ATTN_DENSE = 0, PK_ATTN_SEL = 1, PK_GEMM = 2, PK_COUNT = 3 };
+struct Prof {
+    cudaStream_t st = nullptr;
+    std::vector<cudaEvent_t> ev;
+    std::vector<int> kind;
+    int begin(int k) {
+        cudaEvent_t a, b;
+        if (cudaEventCreate(&a) != cudaSuccess) return -1;
+        if (cudaEventCreate(&b) != cudaSuccess) { cudaEventDestroy(a); return -1; }
+        cudaEventRecord(a, st);
+        ev.push_back(a); ev.push_back(b); kind.push_back(k);
+        return (int)kind.size() - 1;
+    }
+    void end(int i) {
+        if (i >= 0) cudaEventRecord(ev[2 * i + 1], st);
+    }
+    void sums(float* ms, int* n) const {
+        for (int k = 0; k < PK_COUNT; ++k) { ms[k] = 0.f; n[k] = 0; }
+        for (size_t i = 0; i < kind.size(); ++i) {
+            float t = 0.f;
+            cudaEventElapsedTime(&t, ev[2 * i], ev[2 * i + 1]);
+            ms[kind[i]] += t;
+            n[kind[i]] += 1;
+        }
+    }
+    ~Prof() {
+        for (auto e : ev) cudaEventDestroy(e);
+    }
+};
+
 struct Ctx {
     const kvb_config* c;
     const kvb_rope_table* rope;
     Workspace w;
     cudaStream_t st;
     int H, QD, KVD, D, Hq, Hkv, F;
+    Prof* prof = nullptr;
 };
+
+// launch a GEMM, timed when profiling
+kvb_status gemm(const Ctx& x, const GemmParams& p, const uint16_t* A, int64_t lda, const uint16_t* B, int64_t ldb,
+                const uint16_t* B2) {
+    const int i = x.prof ? x.prof->begin(PK_GEMM) : -1;
+    kvb_status s = launch_gemm(p, A, lda, B, ldb, B2, x.st);
+    if (x.prof) x.prof->end(i);
+    return s;
+}
 
 Ctx make_ctx(const kvb_config* c, const kvb_rope_table* rope, const Workspace& w, void* stream) {
     Ctx x;
@@ -218,31 +265,34 @@ kvb_status qkv_rows(const Ctx& x, const kvb_layer_weights* lw, const float* xin,
     p.col_base = 0; p.q_dim = x.QD; p.kv_dim = x.KVD; p.head_dim = x.D;
     p.q_out = q; p.k_out = k; p.v_out = v; p.kv_dst = kv_dst; p.rope_pos = rope_pos;
     p.cos_t = x.rope->cos; p.sin_t = x.rope->sin; p.status = x.w.status;
-    return launch_gemm(p, x.w.a, x.H, lw->w_qkv, x.H, nullptr, x.st);
+    return gemm(x, p, x.w.a, x.H, lw->w_qkv, x.H, nullptr);
 }
 
 // x += attn W_o^T ; x += W_d(silu(W_g n) * W_u n), n = RMSNorm(x)
 kvb_status mlp_rows(const Ctx& x, const kvb_layer_weights* lw, const uint16_t* attn, int64_t m, float* xio) {
     GemmParams p{};
     p.M = m; p.N = x.H; p.K = x.QD; p.epi = EPI_RESID; p.x = xio; p.ldx = x.H; p.status = x.w.status;
-    KVB_TRY(launch_gemm(p, attn, x.QD, lw->w_o, x.QD, nullptr, x.st));
+    KVB_TRY(gemm(x, p, attn, x.QD, lw->w_o, x.QD, nullptr));
     KVB_TRY(launch_rmsnorm(xio, nullptr, m, x.H, lw->mlp_norm, x.c->rms_eps, x.w.a, nullptr, x.st));
     GemmParams g{};
     g.M = m; g.N = x.F; g.K = x.H; g.epi = EPI_SWIGLU; g.out = x.w.h; g.ldo = x.F; g.status = x.w.status;
-    KVB_TRY(launch_gemm(g, x.w.a, x.H, lw->w_gate, x.H, lw->w_up, x.st));
+    KVB_TRY(gemm(x, g, x.w.a, x.H, lw->w_gate, x.H, lw->w_up));
     GemmParams d{};
     d.M = m; d.N = x.H; d.K = x.F; d.epi = EPI_RESID; d.x = xio; d.ldx = x.H; d.status = x.w.status;
-    return launch_gemm(d, x.w.h, x.F, lw->w_down, x.F, nullptr, x.st);
+    return gemm(x, d, x.w.h, x.F, lw->w_down, x.F, nullptr);
 }
 
 kvb_status attn_rows(const Ctx& x, const uint16_t* q, const int32_t* q_idx, const int32_t* kv_lo, int64_t m,
-                     const uint16_t* kc, const uint16_t* vc, int64_t n_kv, uint16_t* out) {
+                     const uint16_t* kc, const uint16_t* vc, int64_t n_kv, uint16_t* out, bool selective = false) {
     AttnParams a{};
     a.q_idx = q_idx; a.kv_lo = kv_lo; a.m = m; a.n_kv = n_kv;
     a.Hq = x.Hq; a.Hkv = x.Hkv; a.D = x.D; a.out = out;
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)x.D));
     a.status = x.w.status;
-    return launch_attn(a, q, kc, vc, x.st);
+    const int i = x.prof ? x.prof->begin(selective ? PK_ATTN_SEL : PK_ATTN_DENSE) : -1;
+    kvb_status s = launch_attn(a, q, kc, vc, x.st);
+    if (x.prof) x.prof->end(i);
+    return s;
 }
 
 // one decoder layer over m rows whose residual is the dense buffer xio [m][H]
@@ -250,7 +300,7 @@ kvb_status attn_rows(const Ctx& x, const uint16_t* q, const int32_t* q_idx, cons
 kvb_status layer(const Ctx& x, const kvb_layer_weights* lw, float* xio, int64_t m, const int32_t* kv_row,
                  const int32_t* rope_pos, const int32_t* kv_lo, uint16_t* kc, uint16_t* vc, int64_t n_kv) {
     KVB_TRY(qkv_rows(x, lw, xio, nullptr, rope_pos, m, x.w.q, kc, vc, kv_row));
-    KVB_TRY(attn_rows(x, x.w.q, kv_row ? kv_row : x.w.ident, kv_lo, m, kc, vc, n_kv, x.w.attn));
+    KVB_TRY(attn_rows(x, x.w.q, kv_row ? kv_row : x.w.ident, kv_lo, m, kc, vc, n_kv, x.w.attn, kv_row != nullptr));
     return mlp_rows(x, lw, x.w.attn, m, xio);
 }
 
@@ -280,6 +330,19 @@ struct Timer {
 };
 
 }  // namespace
+
+static void fill_kernel_times(const Prof& prof, kvb_timings* t, int64_t launches) {
+    float ms[PK_COUNT];
+    int n[PK_COUNT];
+    prof.sums(ms, n);
+    t->attn_dense_ms = ms[PK_ATTN_DENSE];
+    t->attn_sel_ms = ms[PK_ATTN_SEL];
+    t->gemm_ms = ms[PK_GEMM];
+    t->n_attn_dense = n[PK_ATTN_DENSE];
+    t->n_attn_sel = n[PK_ATTN_SEL];
+    t->n_gemm = n[PK_GEMM];
+    t->n_launches = (int32_t)launches;
+}
 
 // ============================================================================ ABI
 
@@ -487,6 +550,10 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
     Workspace w;
     KVB_TRY(carve(cfg, n, ws, ws_bytes, &w));
     Ctx c = make_ctx(cfg, rope, w, stream);
+    Prof prof;
+    prof.st = c.st;
+    if (t) c.prof = &prof;
+    const int64_t launches0 = launch_count();
     Timer tm;
     tm.start(t != nullptr, c.st);
     const int64_t kvd = c.KVD;
@@ -510,6 +577,7 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
         t->total_ms = tm.ms(0, 2);
         t->n_selected = n;
         t->n_rows = n;
+        fill_kernel_times(prof, t, launch_count() - launches0);
     }
     return KVB_OK;
 }
@@ -548,6 +616,10 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
     Workspace w;
     KVB_TRY(carve(cfg, N, ws, ws_bytes, &w));
     Ctx c = make_ctx(cfg, rope, w, stream);
+    Prof prof;
+    prof.st = c.st;
+    if (t) c.prof = &prof;
+    const int64_t launches0 = launch_count();
     const int64_t kvd = c.KVD, rows_c = cache->n_rows;
     auto kc = [&](int l) { return cache->k + (int64_t)l * rows_c * kvd; };
     auto vc = [&](int l) { return cache->v + (int64_t)l * rows_c * kvd; };
@@ -581,7 +653,7 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
                 p.col_base = c.QD; p.q_dim = c.QD; p.kv_dim = c.KVD; p.head_dim = c.D;
                 p.k_out = w.k_fresh; p.rope_pos = w.ident; p.cos_t = rope->cos; p.sin_t = rope->sin;
                 p.status = w.status;
-                KVB_TRY(launch_gemm(p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr, c.st));
+                KVB_TRY(gemm(c, p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr));
                 KVB_TRY(launch_hkvd(w.k_fresh, kvd, kc(lc), kvd, n_ctx, (int)kvd, k, w.sel, w.dev, w.topk, c.st));
             }
             sel = w.sel;
@@ -618,6 +690,7 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
         t->total_ms = tm.ms(0, 5);
         t->n_selected = k;
         t->n_rows = m;
+        fill_kernel_times(prof, t, launch_count() - launches0);
     }
     return KVB_OK;
 }

@@ -327,6 +327,7 @@ kvb_status run(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
     }
     const int64_t grid = (int64_t)nb * p.Hkv;
     kern<<<(unsigned)grid, THREADS, Smem<D>::TOTAL, st>>>(q, k, v, p, nb);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "attention launch");
 }
 

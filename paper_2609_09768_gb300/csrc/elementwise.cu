@@ -184,12 +184,14 @@ kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv
                                                  n_layers, chunk_start, n_chunks, n_ctx, copy_v);
     else
         return fail(KVB_ERR_UNSUPPORTED, "realign: head_dim %d not built", D);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "realign launch");
 }
 
 kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, float* x, cudaStream_t st) {
     if (n <= 0) return KVB_OK;
     embed_kernel<<<grid_for(n * (H / 8), 256), 256, 0, st>>>(embed, tok, n, H, x);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "embed launch");
 }
 
@@ -210,12 +212,14 @@ kvb_status launch_rmsnorm(const float* x, const int32_t* idx, int64_t m, int H, 
             else
                 return fail(KVB_ERR_UNSUPPORTED, "rmsnorm: hidden %d not built", H);
     }
+    count_launch();
     return cuda_ok(cudaGetLastError(), "rmsnorm launch");
 }
 
 kvb_status launch_gather_rows(const float* src, const int32_t* idx, int64_t m, int H, float* dst, cudaStream_t st) {
     if (m <= 0) return KVB_OK;
     gather_rows_kernel<<<grid_for(m * (H / 4), 256), 256, 0, st>>>(src, idx, m, H, dst);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "gather launch");
 }
 
@@ -223,12 +227,14 @@ kvb_status launch_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const 
                           int kv_dim, uint16_t* k_dst, uint16_t* v_dst, cudaStream_t st) {
     if (m <= 0) return KVB_OK;
     scatter_kernel<<<grid_for(m * (kv_dim / 8), 256), 256, 0, st>>>(k_rows, v_rows, dst_idx, m, kv_dim, k_dst, v_dst);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "scatter launch");
 }
 
 kvb_status launch_iota(int32_t* out, int64_t n, int32_t start, cudaStream_t st) {
     if (n <= 0) return KVB_OK;
     iota_kernel<<<grid_for(n, 256), 256, 0, st>>>(out, n, start);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "iota launch");
 }
 
@@ -236,6 +242,7 @@ kvb_status launch_concat_rows(const int32_t* sel, int64_t k, int64_t n_ctx, int6
                               cudaStream_t st) {
     if (k + n_query <= 0) return KVB_OK;
     concat_rows_kernel<<<grid_for(k + n_query, 256), 256, 0, st>>>(sel, k, n_ctx, n_query, rows);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "rows launch");
 }
 

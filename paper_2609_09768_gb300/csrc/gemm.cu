@@ -298,6 +298,7 @@ kvb_status run(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& b2
     }
     const int grid = tiles < num_sms() ? tiles : num_sms();
     kern<<<grid, THREADS, SMEM_BYTES, st>>>(a, b, b2, p);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "gemm launch");
 }
 

@@ -145,9 +145,11 @@ kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t
     const int64_t cap = (int64_t)num_sms() * 16;
     if (blocks > cap) blocks = cap;
     dev_kernel<<<(unsigned)blocks, 256, 0, st>>>(k_fresh, ld_fresh, k_cached, ld_cached, n_ctx, kv_dim, dev_out);
+    count_launch();
     kvb_status s = cuda_ok(cudaGetLastError(), "deviation launch");
     if (s != KVB_OK || k <= 0) return s;
     topk_kernel<<<1, TOPK_THREADS, 0, st>>>(dev_out, n_ctx, k, sel_out);
+    count_launch();
     return cuda_ok(cudaGetLastError(), "top-k launch");
 }
 

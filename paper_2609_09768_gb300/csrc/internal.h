@@ -14,6 +14,9 @@ kvb_status fail(kvb_status s, const char* fmt, ...);
 // KVB_OK, or KVB_ERR_CUDA with the CUDA error text.
 kvb_status cuda_ok(cudaError_t e, const char* what);
 int num_sms();
+// Counts kernels the library launched (for the prefill's launch report).
+void count_launch();
+int64_t launch_count();
 bool aligned16(const void* p);
 
 // Tensor map for a row-major bf16 matrix [rows][cols] (row stride ld elements),

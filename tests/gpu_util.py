@@ -8,6 +8,11 @@ bf16-representable inputs):
     the reference RMS, max <= 2e-2 * rms and mean <= 2e-3 * rms, i.e. the same bar
     applied to a unit-scale signal.  One bf16 rounding of the result alone
     contributes up to 2^-9 (0.2 %) relative per element.
+  * tensors that both sides store in bf16 (q, k, v, caches, re-aligned keys):
+    fp32 and fp64 accumulation can land on opposite sides of a bf16 rounding
+    boundary, so single elements may differ by one bf16 ulp (2^-7 relative at
+    most); the bar is |err| <= 2^-7 |ref| + 1e-3 rms elementwise and mean-abs
+    <= 2e-3 rms.
   * attention outputs: the same bar relative to the RMS of V.  The output is a
     convex combination of value rows; rounding each softmax weight to bf16 (the
     P operand of the P.V product) perturbs it by at most 2^-9 * max|v - out|,
@@ -62,6 +67,16 @@ def assert_close_rel(got, want, what="", max_rel=MAX_ABS, mean_rel=MEAN_ABS, sca
     assert np.all(np.isfinite(np64(got))), f"{what}: non-finite values"
     s = max(e["rms_ref"] if scale is None else scale, 1e-30)
     assert e["max_abs"] <= max_rel * s and e["mean_abs"] <= mean_rel * s, f"{what}: {e}"
+    return e
+
+
+def assert_close_bf16(got, want, what="", mean_rel=MEAN_ABS):
+    g, w = np64(got), np64(want)
+    e = errs(g, w)
+    assert np.all(np.isfinite(g)), f"{what}: non-finite values"
+    s = max(e["rms_ref"], 1e-30)
+    bad = np.abs(g - w) > 2.0 ** -7 * np.abs(w) + 1e-3 * s
+    assert not bad.any() and e["mean_abs"] <= mean_rel * s, f"{what}: {e}, {int(bad.sum())} elements over 1 ulp"
     return e
 
 
