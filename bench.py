@@ -201,7 +201,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     dstarts = torch.tensor(starts, dtype=torch.int32, device=dev)
     kch, vch = workload.chunk_caches(cfg, model, rope, toks[:n_ctx], starts, ws=ws)
     ck = torch.empty(L, N, Hkv, D, dtype=torch.bfloat16, device=dev)
-    cv = torch.empty_like(ck)
+    cv = torch.empty(L, N, Hkv, D, dtype=torch.float16, device=dev)
     fh = torch.empty(nq, H, dtype=torch.float32, device=dev)
     sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
     torch.cuda.synchronize()

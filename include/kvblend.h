@@ -16,7 +16,7 @@
  *    memory of the current CUDA device.  The caller owns all buffers; the library
  *    never allocates or frees device memory.  Scratch memory comes from a caller
  *    workspace whose size kvb_workspace_size() / kvb_hkvd_workspace_size() give.
- *  - bf16 tensors are passed as uint16_t* (raw bfloat16 bits); fp32 as float*.
+ *  - bf16 and fp16 tensors are passed as uint16_t* (raw bits); fp32 as float*.
  *  - All device pointers must be 16-byte aligned.  Matrices are row-major and dense.
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *    Every call is asynchronous on that stream and enqueues no host synchronisation,
@@ -31,9 +31,13 @@
  *
  * Model layout (Llama-3.1 decoder, Sec. 4): hidden H, Hq query heads, Hkv kv heads,
  * head dim D in {64, 128}, MLP dim F, Hq % Hkv == 0 and 128 % (Hq/Hkv) == 0.
- *  - KV cache of one layer: [n_rows][Hkv][D] bf16 for K and for V; a multi-layer
- *    cache is n_layers such blocks back to back.  Row t of the blended cache holds
- *    token t of the concatenated sequence (global position t).
+ *  - KV cache of one layer: [n_rows][Hkv][D] for K and for V; a multi-layer cache
+ *    is n_layers such blocks back to back.  Row t of the blended cache holds token t
+ *    of the concatenated sequence (global position t).  K is bf16.  V holds
+ *    bf16-precision values (the paper's bf16 KV cache) in fp16 containers, so that
+ *    the attention's P.V product runs as an fp16 MMA whose softmax weights are
+ *    rounded to fp16 rather than bf16 (8x smaller rounding error, same speed).
+ *    Converting a bf16 V cache to this layout is exact.
  *  - RoPE is rotate-half (dimension i pairs with i + D/2); tables hold
  *    cos/sin(pos * w_i) in fp32, [max_pos][D/2], computed in double precision.
  */
@@ -96,7 +100,8 @@ typedef struct kvb_rope_table {
     int64_t max_pos;
 } kvb_rope_table;
 
-/* Multi-layer KV cache: k and v are [n_layers][n_rows][Hkv][D] bf16. */
+/* Multi-layer KV cache: k (bf16) and v (fp16, bf16-precision values) are
+ * [n_layers][n_rows][Hkv][D]. */
 typedef struct kvb_kv_cache {
     uint16_t* k;
     uint16_t* v;
@@ -149,7 +154,7 @@ kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos,
  *   k_dst[l][t] = R(chunk_start[c]) k_src[l][t]   (rotation of every head's pairs by
  *                                                  the chunk offset, fp32 math)
  *   v_dst[l][t] = v_src[l][t]                     (skipped when v_src == v_dst or NULL)
- * k_src/v_src are [n_layers][src_rows][Hkv][D] with keys rotated at chunk-local
+ * k_src/v_src are [n_layers][src_rows][Hkv][D] (K bf16, V fp16) with keys rotated at chunk-local
  * positions; k_dst/v_dst are [n_layers][dst_rows][Hkv][D].  In place is allowed
  * (k_src == k_dst, src_rows == dst_rows).  chunk_start: DEVICE int32 [n_chunks+1],
  * ascending, chunk_start[0] == 0, chunk_start[n_chunks] == n_ctx.  The rope table
@@ -185,7 +190,8 @@ kvb_status kvb_hkvd_select(const uint16_t* k_fresh, int64_t ld_fresh,
  *   a[r]   = RMSNorm(x[row_idx[r]]) * attn_norm          (x: fp32 [*][H]; row_idx NULL = r)
  *   q[r]   = RoPE(a[r] W_q^T, rope_pos[r])  -> q_out [m][Hq D] bf16
  *   k[r]   = RoPE(a[r] W_k^T, rope_pos[r])  -> k_out row kv_dst[r] (or r), [*][Hkv D] bf16
- *   v[r]   = a[r] W_v^T                     -> v_out row kv_dst[r] (or r)
+ *   v[r]   = a[r] W_v^T                     -> v_out row kv_dst[r] (or r), fp16 holding
+ *                                              the bf16-rounded value
  * Passing a cache layer as k_out/v_out with kv_dst = the rows' cache indices fuses the
  * KV scatter.  rope_pos: [m] int32 (< rope->max_pos).  Uses tcgen05 tensor cores
  * (bf16 in, fp32 accumulate).  Workspace >= kvb_workspace_size(cfg, m).  Errors:
@@ -212,8 +218,9 @@ kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows,
  *   out[r, j] = sum_{t = lo_r}^{hi_r} softmax_t(q[r, j] . K[t, g] / sqrt(D)) V[t, g],
  *   g = j / (Hq/Hkv), hi_r = q_idx[r], lo_r = kv_lo ? kv_lo[r] : 0.
  * q: [m][Hq][D] bf16 (rotated); q_idx: [m] int32, ascending, < n_kv; kv_lo: [m] or
- * NULL; k_cache/v_cache: one layer, [n_kv][Hkv][D] bf16; out: [m][Hq D] bf16.
- * tcgen05 tensor cores, fp32 softmax.  Errors: INVALID_ARG, UNSUPPORTED. */
+ * NULL; k_cache (bf16) / v_cache (fp16): one layer, [n_kv][Hkv][D]; out: [m][Hq D]
+ * bf16.  tcgen05 tensor cores (Q.K^T bf16, P.V fp16), fp32 softmax.  ws: at least
+ * 256 bytes (device status word).  Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE. */
 kvb_status kvb_sparse_query_attn(const kvb_config* cfg, const uint16_t* q,
                                  const int32_t* q_idx, const int32_t* kv_lo, int64_t m,
                                  const uint16_t* k_cache, const uint16_t* v_cache, int64_t n_kv,
@@ -241,8 +248,8 @@ kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* byt
  *  4. layers >= check_layer: rows S = selected context rows + the n_query query rows,
  *     K/V scattered into the cache before attention over the whole cache;
  *  5. final RMSNorm of the query rows -> final_hidden [n_query][H] fp32.
- * k_chunks/v_chunks: [n_layers][n_ctx][Hkv][D] bf16, each chunk's cache at chunk-local
- * positions (read only).  cache: output blended cache with n_rows >= n_ctx + n_query.
+ * k_chunks/v_chunks: [n_layers][n_ctx][Hkv][D] (K bf16, V fp16), each chunk's cache at
+ * chunk-local positions (read only).  cache: output blended cache with n_rows >= n_ctx + n_query.
  * token_ids: DEVICE int32 [n_ctx + n_query]; chunk_start: DEVICE int32 [n_chunks+1]
  * with chunk_start[n_chunks] == n_ctx.  r in [0, 1]; 1 <= check_layer <= n_layers
  * (check_layer == n_layers means every layer is dense).  forced_sel: DEVICE int32

@@ -15,9 +15,13 @@
 //                MN-major operand, O accumulated in TMEM)
 //   4 softmax warps (thread = row): read S_j from TMEM, mask, online softmax with
 //                a lazily updated running max (O is rescaled only when the max
-//                grows by more than 2^8), write P_j (bf16) to swizzled smem.
+//                grows by more than 2^8), write P_j to swizzled smem.
 // Lazy rescaling keeps the result exact: every term uses the same reference max
 // as the running sum it is divided by.
+// Precision: Q.K^T runs on bf16 operands; P.V runs on fp16 operands - the
+// softmax weights are rounded to fp16 (2^-11 relative instead of bf16's 2^-8),
+// scaled by 2^7 so that they stay in fp16's normal range (p <= 2^15), and the
+// V cache holds bf16-precision values in fp16 containers.
 #include <float.h>
 
 #include "common.cuh"
@@ -30,6 +34,7 @@ constexpr int THREADS = 192;
 constexpr int KT_ROWS = 128;                 // keys per tile
 constexpr uint32_t TMEM_COLS = 512;
 constexpr float RESCALE_LOG2 = 8.0f;
+constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
 
 template <int D>
 struct Smem {
@@ -158,7 +163,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         if (lane == 0 && n_tiles > 0) {
             // ------------------------------------------------ MMA issuer
             constexpr uint32_t IDESC_S = idesc_bf16(128, KT_ROWS, false);
-            constexpr uint32_t IDESC_O = idesc_bf16(128, D, true);
+            constexpr uint32_t IDESC_O = idesc_f16kind(128, D, true, false);   // fp16 P and V
             const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(sK), v0 = smem_u32(sV), p0 = smem_u32(sP);
             bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
             tc_fence_after();
@@ -240,7 +245,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
                 l_run *= alpha;
                 m_run = m_new;
             }
-            const float mref = (m_run == -INFINITY) ? 0.f : m_run * sl2;
+            const float mref = ((m_run == -INFINITY) ? 0.f : m_run * sl2) - P_SHIFT_LOG2;
             uint32_t pk[KT_ROWS / 2];
             float lsum = 0.f;
 #pragma unroll
@@ -248,7 +253,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
                 const float e0 = fast_exp2(fmaf(__uint_as_float(s[c]), sl2, -mref));
                 const float e1 = fast_exp2(fmaf(__uint_as_float(s[c + 1]), sl2, -mref));
                 lsum += e0 + e1;
-                pk[c / 2] = pack_bf16(e0, e1);
+                pk[c / 2] = pack_f16(e0, e1);
             }
             l_run += lsum;
 
@@ -346,7 +351,7 @@ kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k
     const uint64_t kvd = (uint64_t)p.Hkv * p.D;
     s = make_tmap_2d(&tk, k_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
     if (s != KVB_OK) return s;
-    s = make_tmap_2d(&tv, v_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
+    s = make_tmap_2d(&tv, v_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
     if (s != KVB_OK) return s;
     const int64_t nb = (p.m + RPB - 1) / RPB;
     if (nb * p.Hkv > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "attention: too many rows");

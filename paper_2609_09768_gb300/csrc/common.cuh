@@ -5,6 +5,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -19,6 +20,17 @@ namespace kvb {
 KVB_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 KVB_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 KVB_DEV float bf16_to_f(uint16_t v) { return __uint_as_float(((uint32_t)v) << 16); }
+// round-to-nearest-even pack of two floats into fp16x2 (lo in the low half)
+KVB_DEV uint32_t pack_f16(float lo, float hi) {
+    __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+// a value rounded to bf16 precision, stored in an fp16 container (exact for |x| in
+// fp16's normal range): the V cache keeps bf16 values in fp16 so that P.V can run
+// as an fp16 MMA with the softmax weights rounded to fp16
+KVB_DEV uint32_t pack_bf16_as_f16(float lo, float hi) {
+    return pack_f16(__bfloat162float(__float2bfloat16_rn(lo)), __bfloat162float(__float2bfloat16_rn(hi)));
+}
 // round-to-nearest-even pack of two floats (lo in the low half)
 KVB_DEV uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -147,12 +159,15 @@ KVB_DEV void mma_commit(uint64_t* bar) {
                  : "memory");
 }
 
-// Instruction descriptor, kind::f16 with bf16 A/B and fp32 D.
-//  bits 4-5 D format (1 = f32), 7-9 A format (1 = bf16), 10-12 B format (1 = bf16),
+// Instruction descriptor, kind::f16 with fp32 D and A/B both bf16 or both fp16.
+//  bits 4-5 D format (1 = f32), 7-9 A format and 10-12 B format (0 = f16, 1 = bf16),
 //  15 A major (0 = K), 16 B major (0 = K, 1 = MN), 17-22 N>>3, 24-28 M>>4.
+__host__ __device__ constexpr uint32_t idesc_f16kind(uint32_t M, uint32_t N, bool b_mn_major, bool bf16) {
+    return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+           ((N >> 3) << 17) | ((M >> 4) << 24);
+}
 __host__ __device__ constexpr uint32_t idesc_bf16(uint32_t M, uint32_t N, bool b_mn_major) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) | ((N >> 3) << 17) |
-           ((M >> 4) << 24);
+    return idesc_f16kind(M, N, b_mn_major, true);
 }
 
 // Shared-memory matrix descriptor with 128-byte swizzle.

@@ -40,6 +40,16 @@ struct TileMap {
     }
 };
 
+KVB_DEV void store16_bf16_as_f16(uint16_t* dst, const float* v) {
+    uint4 a, b;
+    a.x = pack_bf16_as_f16(v[0], v[1]);   a.y = pack_bf16_as_f16(v[2], v[3]);
+    a.z = pack_bf16_as_f16(v[4], v[5]);   a.w = pack_bf16_as_f16(v[6], v[7]);
+    b.x = pack_bf16_as_f16(v[8], v[9]);   b.y = pack_bf16_as_f16(v[10], v[11]);
+    b.z = pack_bf16_as_f16(v[12], v[13]); b.w = pack_bf16_as_f16(v[14], v[15]);
+    reinterpret_cast<uint4*>(dst)[0] = a;
+    reinterpret_cast<uint4*>(dst)[1] = b;
+}
+
 KVB_DEV void store16_bf16(uint16_t* dst, const float* v) {
     uint4 a, b;
     a.x = pack_bf16(v[0], v[1]);   a.y = pack_bf16(v[2], v[3]);
@@ -225,7 +235,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                                 float y[16];
 #pragma unroll
                                 for (int i = 0; i < 16; ++i) y[i] = __uint_as_float(x1[i]);
-                                store16_bf16(outp + c * 16, y);
+                                store16_bf16_as_f16(outp + c * 16, y);
                             }
                         }
                     }

@@ -22,7 +22,8 @@ bool aligned16(const void* p);
 // Tensor map for a row-major bf16 matrix [rows][cols] (row stride ld elements),
 // box [box_rows][box_cols], 128-byte swizzle.
 kvb_status make_tmap_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld,
-                        uint32_t box_cols, uint32_t box_rows);
+                        uint32_t box_cols, uint32_t box_rows,
+                        CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16);
 // Tensor map over [d2][d1][d0] bf16 (dense), box [b2][b1][b0], 128-byte swizzle.
 kvb_status make_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
                         uint32_t b0, uint32_t b1, uint32_t b2);

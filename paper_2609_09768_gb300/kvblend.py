@@ -183,9 +183,9 @@ class Model:
 
 
 def kv_cache_struct(k: torch.Tensor, v: torch.Tensor) -> KVCache:
-    """k, v: [L][n_rows][Hkv][D] bf16."""
+    """k: [L][n_rows][Hkv][D] bf16; v: same shape, fp16 (bf16-precision values)."""
     assert k.shape == v.shape and k.dim() == 4
-    return KVCache(_ptr(k, torch.bfloat16, "cache k"), _ptr(v, torch.bfloat16, "cache v"), k.shape[1], k.shape[0])
+    return KVCache(_ptr(k, torch.bfloat16, "cache k"), _ptr(v, torch.float16, "cache v"), k.shape[1], k.shape[0])
 
 
 # ---------------------------------------------------------------------------------- workspace
@@ -212,8 +212,8 @@ def device_status(ws: torch.Tensor) -> int:
 def rope_realign(cfg: Config, rope: RopeTable, k_src, v_src, k_dst, v_dst, layer_begin: int, layer_end: int,
                  chunk_start: torch.Tensor, n_ctx: int) -> None:
     _call("kvb_rope_realign", C.byref(cfg), C.byref(rope.struct), _ptr(k_src, torch.bfloat16, "k_src"),
-          _ptr(v_src, torch.bfloat16, "v_src"), k_src.shape[1], _ptr(k_dst, torch.bfloat16, "k_dst"),
-          _ptr(v_dst, torch.bfloat16, "v_dst"), k_dst.shape[1], layer_begin, layer_end,
+          _ptr(v_src, torch.float16, "v_src"), k_src.shape[1], _ptr(k_dst, torch.bfloat16, "k_dst"),
+          _ptr(v_dst, torch.float16, "v_dst"), k_dst.shape[1], layer_begin, layer_end,
           _ptr(chunk_start, torch.int32, "chunk_start"), chunk_start.numel() - 1, n_ctx, _stream())
 
 
@@ -237,22 +237,22 @@ def gather_rmsnorm_qkv(cfg: Config, lw: LayerWeights, rope: RopeTable, x: torch.
                        q_out, k_out, v_out, kv_dst, ws: torch.Tensor) -> None:
     _call("kvb_gather_rmsnorm_qkv", C.byref(cfg), C.byref(lw), C.byref(rope.struct), _ptr(x, torch.float32, "x"),
           _ptr(row_idx, torch.int32, "row_idx"), _ptr(rope_pos, torch.int32, "rope_pos"), m,
-          _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"), _ptr(v_out, torch.bfloat16, "v_out"),
+          _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"), _ptr(v_out, torch.float16, "v_out"),
           _ptr(kv_dst, torch.int32, "kv_dst"), _ptr(ws), ws.numel(), _stream())
 
 
 def kv_scatter(k_rows, v_rows, dst_idx, k_dst, v_dst) -> None:
     m = dst_idx.numel()
     kv_dim = k_rows[0].numel() if m else 8
-    _call("kvb_kv_scatter", _ptr(k_rows, torch.bfloat16, "k_rows"), _ptr(v_rows, torch.bfloat16, "v_rows"),
+    _call("kvb_kv_scatter", _ptr(k_rows, torch.bfloat16, "k_rows"), _ptr(v_rows, torch.float16, "v_rows"),
           _ptr(dst_idx, torch.int32, "dst_idx"), m, kv_dim, _ptr(k_dst, torch.bfloat16, "k_dst"),
-          _ptr(v_dst, torch.bfloat16, "v_dst"), k_dst.shape[0], _stream())
+          _ptr(v_dst, torch.float16, "v_dst"), k_dst.shape[0], _stream())
 
 
 def sparse_query_attn(cfg: Config, q, q_idx, kv_lo, k_cache, v_cache, out, ws: torch.Tensor) -> None:
     _call("kvb_sparse_query_attn", C.byref(cfg), _ptr(q, torch.bfloat16, "q"), _ptr(q_idx, torch.int32, "q_idx"),
           _ptr(kv_lo, torch.int32, "kv_lo"), q_idx.numel(), _ptr(k_cache, torch.bfloat16, "k_cache"),
-          _ptr(v_cache, torch.bfloat16, "v_cache"), k_cache.shape[0], _ptr(out, torch.bfloat16, "out"), _ptr(ws),
+          _ptr(v_cache, torch.float16, "v_cache"), k_cache.shape[0], _ptr(out, torch.bfloat16, "out"), _ptr(ws),
           ws.numel(), _stream())
 
 
@@ -278,7 +278,7 @@ def selective_prefill(cfg: Config, model: Model, rope: RopeTable, k_chunks, v_ch
     cache = kv_cache_struct(cache_k, cache_v)
     t = Timings()
     _call("kvb_selective_prefill", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct),
-          _ptr(k_chunks, torch.bfloat16, "k_chunks"), _ptr(v_chunks, torch.bfloat16, "v_chunks"), C.byref(cache),
+          _ptr(k_chunks, torch.bfloat16, "k_chunks"), _ptr(v_chunks, torch.float16, "v_chunks"), C.byref(cache),
           _ptr(token_ids, torch.int32, "token_ids"), _ptr(chunk_start, torch.int32, "chunk_start"),
           (chunk_start.numel() - 1) if chunk_start is not None else 0, n_ctx, n_query, r, check_layer,
           _ptr(forced_sel, torch.int32, "forced_sel"), forced_sel.numel() if forced_sel is not None else 0,

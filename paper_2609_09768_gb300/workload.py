@@ -33,12 +33,12 @@ def chunk_layout(chunk_starts: List[int], device="cuda"):
 
 def chunk_caches(cfg: kvb.Config, model: kvb.Model, rope: kvb.RopeTable, ctx_tokens: torch.Tensor,
                  chunk_starts: List[int], ws: Optional[torch.Tensor] = None):
-    """Per-chunk caches [L][n_ctx][Hkv][D] (keys at chunk-local positions)."""
+    """Per-chunk caches [L][n_ctx][Hkv][D] (keys at chunk-local positions; K bf16, V fp16)."""
     n_ctx = chunk_starts[-1]
     L = cfg.n_layers
     dev = ctx_tokens.device
     k = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.bfloat16, device=dev)
-    v = torch.empty_like(k)
+    v = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.float16, device=dev)
     pos, lo = chunk_layout(chunk_starts, dev)
     kvb.full_prefill(cfg, model, rope, k, v, ctx_tokens, rope_pos=pos, kv_lo=lo, ws=ws)
     return k, v

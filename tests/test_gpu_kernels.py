@@ -37,12 +37,12 @@ def test_realign_matches_oracle(kvb, shape, starts):
     cfg = kvb.config(shape)
     n_ctx, L, Hkv, D = starts[-1], shape.n_layers, shape.n_kv_heads, shape.head_dim
     k_src = synth.randn_bf16((L, n_ctx, Hkv, D), 101)
-    v_src = synth.randn_bf16((L, n_ctx, Hkv, D), 102)
+    v_src = synth.randn_bf16((L, n_ctx, Hkv, D), 102).to(torch.float16)
     rope = kvb.RopeTable(cfg, n_ctx)
     cs = dev(torch.tensor(starts, dtype=torch.int32))
     rows = n_ctx + 13
     k_dst = torch.zeros(L, rows, Hkv, D, dtype=torch.bfloat16, device="cuda")
-    v_dst = torch.zeros_like(k_dst)
+    v_dst = torch.zeros(L, rows, Hkv, D, dtype=torch.float16, device="cuda")
     kvb.rope_realign(cfg, rope, dev(k_src), dev(v_src), k_dst, v_dst, 0, L, cs, n_ctx)
     torch.cuda.synchronize()
     ref = blend.realign(Shape.of(shape, act_bf16=True), np64(k_src), starts)
@@ -115,7 +115,7 @@ def test_gather_rmsnorm_qkv_matches_oracle(kvb, shape, m, n_src):
     rope = kvb.RopeTable(cfg, max_pos)
     q = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
     kc = torch.zeros(n_cache, shape.kv_dim, dtype=torch.bfloat16, device="cuda")
-    vc = torch.zeros_like(kc)
+    vc = torch.zeros(n_cache, shape.kv_dim, dtype=torch.float16, device="cuda")
     ws = kvb.workspace(cfg, m)
     kvb.gather_rmsnorm_qkv(cfg, kvb.layer_struct(lwd), rope, dev(x), dev(row_idx), dev(rope_pos), m, q, kc, vc,
                            dev(kv_dst), ws)
@@ -138,7 +138,7 @@ def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
     m = len(q_rows)
     q = synth.randn_bf16((m, shape.n_q_heads, shape.head_dim), seed)
     k = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 1)
-    v = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 2)
+    v = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 2).to(torch.float16)
     qi = torch.tensor(q_rows, dtype=torch.int32)
     lo = None if kv_lo is None else torch.tensor(kv_lo, dtype=torch.int32)
     out = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
@@ -204,14 +204,14 @@ def test_mlp_rows_matches_oracle(kvb, shape, m):
 def test_kv_scatter_bit_exact(kvb, m, kv_dim, n_dst):
     g = torch.Generator().manual_seed(m)
     kr = synth.randn_bf16((m, kv_dim), 401)
-    vr = synth.randn_bf16((m, kv_dim), 402)
+    vr = synth.randn_bf16((m, kv_dim), 402).to(torch.float16)
     idx = torch.randperm(n_dst, generator=g)[:m].to(torch.int32)
     kd = torch.zeros(n_dst, kv_dim, dtype=torch.bfloat16, device="cuda")
-    vd = torch.zeros_like(kd)
+    vd = torch.zeros(n_dst, kv_dim, dtype=torch.float16, device="cuda")
     kvb.kv_scatter(dev(kr), dev(vr), dev(idx), kd, vd)
     torch.cuda.synchronize()
     want_k = torch.zeros(n_dst, kv_dim, dtype=torch.bfloat16)
-    want_v = torch.zeros_like(want_k)
+    want_v = torch.zeros(n_dst, kv_dim, dtype=torch.float16)
     want_k[idx.long()] = kr
     want_v[idx.long()] = vr
     assert torch.equal(kd.cpu(), want_k) and torch.equal(vd.cpu(), want_v)

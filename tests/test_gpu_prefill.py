@@ -57,7 +57,7 @@ class Case:
         self.dtoks = self.toks.cuda()
         self.dstarts = torch.tensor(self.starts, dtype=torch.int32, device="cuda")
         self.kch = torch.from_numpy(self.cc["k"]).to(torch.bfloat16).cuda()
-        self.vch = torch.from_numpy(self.cc["v"]).to(torch.bfloat16).cuda()
+        self.vch = torch.from_numpy(self.cc["v"]).to(torch.bfloat16).to(torch.float16).cuda()
         self.ws = kvb.workspace(self.cfg, self.N)
 
     def fp64_gap(self, got, ref64, what):
@@ -69,7 +69,7 @@ class Case:
     def new_cache(self):
         k = torch.zeros(self.shape.n_layers, self.N, self.shape.n_kv_heads, self.shape.head_dim,
                         dtype=torch.bfloat16, device="cuda")
-        return k, torch.zeros_like(k)
+        return k, torch.zeros(k.shape, dtype=torch.float16, device="cuda")
 
 
 _CASES = {}
