@@ -288,6 +288,13 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
  * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */
 kvb_status kvb_device_status(void* ws, size_t ws_bytes, void* stream, int32_t* code_out);
 
+/* Exercise the bounded-wait path (for tests; the paper has no counterpart): launch one
+ * CTA that waits on an mbarrier nothing completes, giving up after limit_ns
+ * (1000 <= limit_ns <= 4e9) and recording KVB_ERR_TIMEOUT in the status word of `ws`
+ * exactly as a stalled pipeline in the GEMM or attention kernels would.  The CUDA
+ * context stays usable.  Errors: INVALID_ARG. */
+kvb_status kvb_debug_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

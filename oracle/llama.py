@@ -24,6 +24,12 @@ model holds in bf16 - the RMSNorm outputs that feed a linear layer, q/k/v after
 RoPE (k and v are the KV cache), the attention output, the SwiGLU product and
 the re-aligned cached keys - and keeps everything else (accumulation, softmax,
 the residual stream) in float64.  Without it every tensor stays float64.
+
+`Shape.accum32` makes the linear layers accumulate in float32 instead.  It is
+not the reference: it is a second correct implementation whose distance from the
+float64 one measures how far two faithful implementations of the same bf16 model
+drift apart through accumulation rounding alone (the floor any fp32-accumulating
+kernel is judged against).
 """
 from __future__ import annotations
 
@@ -51,13 +57,15 @@ class Shape:
     rs_high: float = 4.0
     rs_orig_ctx: int = 8192
     act_bf16: bool = False
+    accum32: bool = False
 
     @staticmethod
-    def of(s, act_bf16: bool = False) -> "Shape":
+    def of(s, act_bf16: bool = False, accum32: bool = False) -> "Shape":
         """Copy the fields from any object that has them (e.g. a ModelShape)."""
         return Shape(s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.mlp_dim,
                      float(s.rms_eps), float(s.rope_theta), bool(s.rope_llama3),
-                     float(s.rs_factor), float(s.rs_low), float(s.rs_high), int(s.rs_orig_ctx), act_bf16)
+                     float(s.rs_factor), float(s.rs_low), float(s.rs_high), int(s.rs_orig_ctx), act_bf16,
+                     accum32)
 
 
 def as64(a) -> np.ndarray:
@@ -140,8 +148,11 @@ def rmsnorm(x: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
     return x / np.sqrt(ms + eps) * as64(g)
 
 
-def linear(x: np.ndarray, w: np.ndarray) -> np.ndarray:
-    """y = x W^T with W stored [out_features, in_features]."""
+def linear(x: np.ndarray, w: np.ndarray, accum32: bool = False) -> np.ndarray:
+    """y = x W^T with W stored [out_features, in_features] (float32 products and sums
+    when accum32)."""
+    if accum32:
+        return (np.asarray(x, np.float32) @ np.asarray(as64(w), np.float32).T).astype(F64)
     return as64(x) @ as64(w).T
 
 
@@ -193,7 +204,7 @@ def qkv_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> tuple[np.ndarray, n
     """RMSNorm -> QKV projection -> RoPE at `rope_pos`.  Returns q [m,Hq,D], k, v [m,Hkv,D]."""
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
     n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
-    qkv = linear(n1, lw["w_qkv"])
+    qkv = linear(n1, lw["w_qkv"], s.accum32)
     m = x.shape[0]
     q = qkv[:, : Hq * D].reshape(m, Hq, D)
     k = qkv[:, Hq * D: (Hq + Hkv) * D].reshape(m, Hkv, D)
@@ -207,17 +218,17 @@ def k_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> np.ndarray:
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
     n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
     wk = as64(lw["w_qkv"])[Hq * D: (Hq + Hkv) * D]
-    k = (n1 @ wk.T).reshape(x.shape[0], Hkv, D)
+    k = linear(n1, wk, s.accum32).reshape(x.shape[0], Hkv, D)
     c, sn = rope_cos_sin(s, rope_pos)
     return act(s, apply_rope(k, c, sn))
 
 
 def attn_out_mlp(s: Shape, lw: dict, x: np.ndarray, attn: np.ndarray) -> np.ndarray:
     """x + O-proj(attn), then + SwiGLU MLP of its RMSNorm.  attn: [m, Hq*D]."""
-    h = as64(x) + linear(attn, lw["w_o"])
+    h = as64(x) + linear(attn, lw["w_o"], s.accum32)
     n2 = act(s, rmsnorm(h, lw["mlp_norm"], s.rms_eps))
-    a = act(s, silu(linear(n2, lw["w_gate"])) * linear(n2, lw["w_up"]))
-    return h + linear(a, lw["w_down"])
+    a = act(s, silu(linear(n2, lw["w_gate"], s.accum32)) * linear(n2, lw["w_up"], s.accum32))
+    return h + linear(a, lw["w_down"], s.accum32)
 
 
 def layer_rows(s: Shape, lw: dict, x: np.ndarray, row_idx, rope_pos, k_cache: np.ndarray,

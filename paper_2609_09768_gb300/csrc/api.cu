@@ -695,6 +695,13 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
     return KVB_OK;
 }
 
+kvb_status kvb_debug_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
+    g_err[0] = 0;
+    if (!ws || ws_bytes < 256 || limit_ns < 1000 || limit_ns > 4000000000ll)
+        return fail(KVB_ERR_INVALID_ARG, "debug wait: bad workspace or limit");
+    return launch_wait_timeout(static_cast<int*>(ws), (uint64_t)limit_ns, static_cast<cudaStream_t>(stream));
+}
+
 kvb_status kvb_device_status(void* ws, size_t ws_bytes, void* stream, int32_t* code_out) {
     g_err[0] = 0;
     if (!ws || ws_bytes < 256 || !code_out) return fail(KVB_ERR_INVALID_ARG, "device status: bad arguments");

@@ -84,14 +84,15 @@ KVB_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Wait until the phase with the given parity has completed.  Gives up after
 // kWaitLimitNs (or as soon as another thread of the CTA has given up, signalled
 // through *abort), records KVB_ERR_TIMEOUT and returns false.
-KVB_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* status) {
+KVB_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* status,
+                       uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
             if (*abort) return false;
-            if (globaltimer() - t0 > kWaitLimitNs) {
+            if (globaltimer() - t0 > limit_ns) {
                 *abort = 1;
                 set_status(status, KVB_ERR_TIMEOUT);
                 return false;

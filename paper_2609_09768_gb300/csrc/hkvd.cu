@@ -133,7 +133,28 @@ topk_kernel(const float* __restrict__ dev, int64_t n, int64_t k, int32_t* __rest
     }
 }
 
+// A wait that nothing completes: the bounded mbarrier wait gives up after limit_ns
+// and records KVB_ERR_TIMEOUT (test hook for the kernels' timeout path).
+__global__ void wait_timeout_kernel(int* status, uint64_t limit_ns) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    mbar_wait(&bar, 0, &abort_flag, status, limit_ns);
+    __syncthreads();
+}
+
 }  // namespace
+
+kvb_status launch_wait_timeout(int* status, uint64_t limit_ns, cudaStream_t st) {
+    wait_timeout_kernel<<<1, 32, 0, st>>>(status, limit_ns);
+    count_launch();
+    return cuda_ok(cudaGetLastError(), "wait-timeout launch");
+}
 
 size_t hkvd_ws_bytes(int64_t) { return 0; }
 

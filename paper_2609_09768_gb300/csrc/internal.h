@@ -95,6 +95,8 @@ kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t
                        int64_t n_ctx, int kv_dim, int64_t k, int32_t* sel_out, float* dev_out, void* scratch,
                        cudaStream_t st);
 
+kvb_status launch_wait_timeout(int* status, uint64_t limit_ns, cudaStream_t st);
+
 // ---------------------------------------------------------------- workspace
 // Layout of a caller workspace for up to n rows.
 struct Workspace {

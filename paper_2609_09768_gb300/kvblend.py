@@ -89,6 +89,7 @@ _SIGS = {
     "kvb_full_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), P(KVCache), c_vp, c_i64, c_vp, c_vp,
                                  c_vp, c_i64, P(Timings), c_vp, c_sz, c_vp]),
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
+    "kvb_debug_wait_timeout": (c_i32, [c_vp, c_sz, c_i64, c_vp]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -199,6 +200,10 @@ def workspace_size(cfg: Config, n_rows: int) -> int:
 def workspace(cfg: Config, n_rows: int, device="cuda") -> torch.Tensor:
     """A zeroed workspace (the zeroed head is the device status word)."""
     return torch.zeros(workspace_size(cfg, n_rows), dtype=torch.uint8, device=device)
+
+
+def debug_wait_timeout(ws: torch.Tensor, limit_ns: int) -> None:
+    _call("kvb_debug_wait_timeout", _ptr(ws), ws.numel(), limit_ns, _stream())
 
 
 def device_status(ws: torch.Tensor) -> int:

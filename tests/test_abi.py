@@ -86,6 +86,7 @@ def test_host_validation_rejects_bad_arguments(kvb):
     mw = kvb.ModelStruct()
     assert L.kvb_selective_prefill(C.byref(cfg), C.byref(mw), None, None, None, None, None, None, 1, 10, 2, 1.5, 1,
                                    None, 0, None, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+    assert L.kvb_debug_wait_timeout(None, 0, 10**6, None) == kvb.KVB_ERR_INVALID_ARG
     # empty inputs are valid no-ops
     assert L.kvb_kv_scatter(None, None, None, 0, 128, None, None, 4, None) == kvb.KVB_OK
     assert L.kvb_hkvd_select(None, 128, None, 128, 0, 128, 0, None, None, None, 0, None) == kvb.KVB_OK

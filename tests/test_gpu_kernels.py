@@ -215,3 +215,21 @@ def test_kv_scatter_bit_exact(kvb, m, kv_dim, n_dst):
     want_k[idx.long()] = kr
     want_v[idx.long()] = vr
     assert torch.equal(kd.cpu(), want_k) and torch.equal(vd.cpu(), want_v)
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(kvb):
+    """A wait that nothing completes gives up after its limit and reports KVB_ERR_TIMEOUT
+    through the status word; the context stays usable and the word is cleared on read."""
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    assert kvb.device_status(ws) == kvb.KVB_OK
+    kvb.debug_wait_timeout(ws, 5_000_000)          # 5 ms
+    assert kvb.device_status(ws) == kvb.KVB_ERR_TIMEOUT
+    assert kvb.device_status(ws) == kvb.KVB_OK       # cleared
+    # the device still runs the real kernels correctly afterwards
+    kr = synth.randn_bf16((4, 128), 7)
+    idx = torch.tensor([3, 0, 5, 1], dtype=torch.int32)
+    kd = torch.zeros(6, 128, dtype=torch.bfloat16, device="cuda")
+    vd = torch.zeros(6, 128, dtype=torch.float16, device="cuda")
+    kvb.kv_scatter(dev(kr), dev(kr.to(torch.float16)), dev(idx), kd, vd)
+    torch.cuda.synchronize()
+    assert torch.equal(kd.cpu()[idx.long()], kr)

@@ -424,3 +424,21 @@ def test_bf16_storage_mode_rounds_only_stored_activations():
     cc = blend.chunk_caches(s16, m["layers_np"], x0[:20], starts)
     re = blend.realign(s16, cc["k"], starts)
     assert np.array_equal(llama.bf16_round(re), re)
+
+
+def test_accum32_is_a_float32_accumulation_of_the_same_model():
+    """accum32 changes only the accumulation precision of the linear layers: it agrees with
+    a float32 torch matmul and with the float64 result to float32 accuracy."""
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((9, 64))
+    w = rng.standard_normal((33, 64)) * 0.02
+    y32 = llama.linear(x, w, accum32=True)
+    ref32 = (torch.as_tensor(x, dtype=torch.float32) @ torch.as_tensor(w, dtype=torch.float32).T).double().numpy()
+    assert rel(y32, ref32) < 1e-6
+    assert 0 < rel(y32, llama.linear(x, w)) < 1e-6
+    shape = MINI.with_layers(2)
+    m = model(shape)
+    x0 = blend.embed_rows(m["embed"], synth.make_tokens(shape, 20, 1).numpy())
+    a = blend.full_prefill(Shape.of(shape, act_bf16=True), m["layers_np"], x0)["x"]
+    b = blend.full_prefill(Shape.of(shape, act_bf16=True, accum32=True), m["layers_np"], x0)["x"]
+    assert 0 < rel(a, b) < 1e-2
