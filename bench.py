@@ -33,6 +33,22 @@ sys.path.insert(0, ROOT)
 
 METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % of bf16 peak"
 
+# DRAM bytes (read + write) per launch of the selective-layer attention at this workload's
+# size (18,713 rows over a 124,032-row cache), from the ncu capture summarised in
+# profiles/attn_kernel_sparse_m18713_nkv124032.md; valid only for the kernel sources it
+# was taken on (sha1 prefixes of attn.cu and common.cuh), otherwise reported as null.
+ATTN_TRAFFIC = {"bytes": 8.171988e9 + 0.141541e9, "sha1": {"attn.cu": "1f315e88dfd7", "common.cuh": "375ffc0357ed"}}
+
+
+def attn_traffic():
+    import hashlib
+    d = os.path.join(ROOT, "paper_2609_09768_gb300", "csrc")
+    for f, h in ATTN_TRAFFIC["sha1"].items():
+        with open(os.path.join(d, f), "rb") as fh:
+            if hashlib.sha1(fh.read()).hexdigest()[:12] != h:
+                return None
+    return ATTN_TRAFFIC["bytes"]
+
 
 def parse():
     ap = argparse.ArgumentParser()
@@ -264,7 +280,8 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     achieved = per_launch_flop / (per_launch_ms * 1e-3) / 1e12
     roofline = {"kernel": dom_name, "bound": "tensor", "achieved": round(achieved, 2),
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": round(achieved / pk["bf16_sustained"], 4),
-                "traffic": None, "peak_source": f"{pk['source']} bf16 sustained",
+                "traffic": attn_traffic() if dom_name == "attn_selective" else None,
+                "peak_source": f"{pk['source']} bf16 sustained",
                 "flop_per_launch": per_launch_flop, "ms_per_launch": round(per_launch_ms, 4)}
 
     # the library's own dense r = 1.0 prefill of the same request
