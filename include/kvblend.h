@@ -204,6 +204,30 @@ kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights
                                   const int32_t* kv_dst,
                                   void* ws, size_t ws_bytes, void* stream);
 
+/* Allocation-free variant of kvb_gather_rmsnorm_qkv (the paper has no counterpart:
+ * this serves callers, not the method).  Some callers cannot hand the library any
+ * device memory of their own - e.g. a plugin inside a serving process whose memory
+ * pool owns all device memory, or a hot loop that must never enter an allocator -
+ * so the scratch this step needs (the m normalised bf16 rows that feed the GEMM)
+ * lives in a fixed array inside the library, KVB_NOALLOC_MAX_ELEMS bf16 values
+ * (8 MiB) that every GPU loading the library holds until the process exits.
+ * Arguments and results are those of kvb_gather_rmsnorm_qkv without the workspace;
+ * status_out (DEVICE int32, zeroed by the caller, or NULL) receives KVB_ERR_TIMEOUT
+ * if a bounded wait in the GEMM runs out.  m * hidden above KVB_NOALLOC_MAX_ELEMS is
+ * rejected with INVALID_ARG.  No memory is allocated or freed.  The first call on a
+ * device looks the array's address up (cudaGetSymbolAddress) for that device, so make
+ * it before any stream capture.  Every call reuses the same array (nothing in it has
+ * to start at zero: each call overwrites the rows it reads); calls whose kernels
+ * overlap on the GPU, e.g. on unordered streams, race on it.  Errors: INVALID_ARG,
+ * UNSUPPORTED, CUDA. */
+#define KVB_NOALLOC_MAX_ELEMS (4 * 1024 * 1024)
+kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, const kvb_layer_weights* w,
+                                          const kvb_rope_table* rope,
+                                          const float* x, const int32_t* row_idx,
+                                          const int32_t* rope_pos, int64_t m,
+                                          uint16_t* q_out, uint16_t* k_out, uint16_t* v_out,
+                                          const int32_t* kv_dst, int32_t* status_out, void* stream);
+
 /* KV scatter (Sec. 3.4: recomputed entries replace the cached ones): for r < m,
  *   k_dst[dst_idx[r]] = k_rows[r], v_dst[dst_idx[r]] = v_rows[r]   (kv_dim elements)
  * dst_idx values must be distinct and < n_dst_rows (bit copy, order irrelevant).

@@ -78,6 +78,8 @@ _SIGS = {
     "kvb_hkvd_select": (c_i32, [c_vp, c_i64, c_vp, c_i64, c_i64, c_i32, c_i64, c_vp, c_vp, c_vp, c_sz, c_vp]),
     "kvb_gather_rmsnorm_qkv": (c_i32, [P(Config), P(LayerWeights), P(RopeTableStruct), c_vp, c_vp, c_vp, c_i64,
                                        c_vp, c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]),
+    "kvb_gather_rmsnorm_qkv_noalloc": (c_i32, [P(Config), P(LayerWeights), P(RopeTableStruct), c_vp, c_vp, c_vp,
+                                               c_i64, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
     "kvb_kv_scatter": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i32, c_vp, c_vp, c_i64, c_vp]),
     "kvb_sparse_query_attn": (c_i32, [P(Config), c_vp, c_vp, c_vp, c_i64, c_vp, c_vp, c_i64, c_vp, c_vp, c_sz,
                                       c_vp]),
@@ -244,6 +246,20 @@ def gather_rmsnorm_qkv(cfg: Config, lw: LayerWeights, rope: RopeTable, x: torch.
           _ptr(row_idx, torch.int32, "row_idx"), _ptr(rope_pos, torch.int32, "rope_pos"), m,
           _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"), _ptr(v_out, torch.float16, "v_out"),
           _ptr(kv_dst, torch.int32, "kv_dst"), _ptr(ws), ws.numel(), _stream())
+
+
+NOALLOC_MAX_ELEMS = 4 * 1024 * 1024
+
+
+def gather_rmsnorm_qkv_noalloc(cfg: Config, lw: LayerWeights, rope: RopeTable, x: torch.Tensor, row_idx, rope_pos,
+                               m: int, q_out, k_out, v_out, kv_dst, status_out: Optional[torch.Tensor] = None) -> None:
+    """kvb_gather_rmsnorm_qkv without a workspace: the library's fixed scratch holds the
+    normalised rows (m * hidden <= NOALLOC_MAX_ELEMS), for callers that cannot allocate."""
+    _call("kvb_gather_rmsnorm_qkv_noalloc", C.byref(cfg), C.byref(lw), C.byref(rope.struct),
+          _ptr(x, torch.float32, "x"), _ptr(row_idx, torch.int32, "row_idx"), _ptr(rope_pos, torch.int32, "rope_pos"),
+          m, _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"),
+          _ptr(v_out, torch.float16, "v_out"), _ptr(kv_dst, torch.int32, "kv_dst"),
+          _ptr(status_out, torch.int32, "status_out"), _stream())
 
 
 def kv_scatter(k_rows, v_rows, dst_idx, k_dst, v_dst) -> None:
