@@ -1,0 +1,242 @@
+"""Parity at the headline workload's full sizes (124,032-token request, Llama-3.1-8B
+shapes), in the launch configurations the benchmark times.  The kernels run on the
+whole problem; the oracle recomputes sampled outputs one row at a time.  The
+32-layer prefill is checked through properties that hold at any size."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import blend, llama
+from oracle.llama import Shape
+from paper_2609_09768_gb300 import synth, workload
+from tests.gpu_util import assert_close_abs, assert_close_bf16, assert_close_rel, np64
+
+pytestmark = pytest.mark.gpu
+
+SHAPE = synth.LLAMA8B
+WL = synth.WORKLOADS["l8b_124k"]
+N, N_CTX = WL.n_total, WL.n_ctx
+M_SEL = 18585 + WL.n_query          # rows a selective layer recomputes at r = 0.15
+
+
+@pytest.fixture(scope="module")
+def kvb():
+    from paper_2609_09768_gb300 import kvblend
+    kvblend.lib()
+    return kvblend
+
+
+def gen(seed):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    return g
+
+
+def sample_rows(m, k=48, seed=0):
+    rng = np.random.default_rng(seed)
+    s = np.unique(np.concatenate([[0, 1, m // 2, m - 2, m - 1], rng.choice(m, size=k, replace=False)]))
+    return s
+
+
+@pytest.mark.parametrize("mode", ["selective", "dense"])
+def test_attention_full_size_sampled_rows(kvb, mode):
+    cfg = kvb.config(SHAPE)
+    g = gen(1)
+    if mode == "dense":
+        rows = torch.arange(N, dtype=torch.int32, device="cuda")
+    else:
+        perm = torch.randperm(N_CTX, generator=g, device="cuda")[: M_SEL - WL.n_query]
+        rows = torch.cat([torch.sort(perm).values,
+                          torch.arange(N_CTX, N, device="cuda")]).to(torch.int32)
+    m = rows.numel()
+    q = torch.randn(m, SHAPE.n_q_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
+    k = torch.randn(N, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
+    v = torch.randn(N, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16).to(torch.float16)
+    out = torch.empty(m, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    kvb.sparse_query_attn(cfg, q, rows, None, k, v, out, ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    smp = sample_rows(m)
+    ri = rows.cpu().numpy()
+    ref = llama.attention_rows(Shape.of(SHAPE), np64(q.cpu()[smp]), np64(k.cpu()), np64(v.cpu()), ri[smp])
+    vs = float(np.sqrt(np.mean(np64(v.cpu()) ** 2)))
+    e = assert_close_rel(out.cpu()[smp], ref.reshape(len(smp), -1), f"{mode} attention at full size", scale=vs)
+    print(mode, m, e)
+
+
+@pytest.mark.parametrize("m", [M_SEL, N])
+def test_qkv_and_mlp_full_size_sampled_rows(kvb, m):
+    cfg = kvb.config(SHAPE)
+    s = Shape.of(SHAPE, act_bf16=True)
+    lw_cpu = synth.make_layer_weights(SHAPE, 3, seed=0)
+    lw = {kk: vv.cuda() for kk, vv in lw_cpu.items()}
+    lws = kvb.layer_struct(lw)
+    g = gen(2)
+    x_all = torch.randn(N, SHAPE.hidden, generator=g, device="cuda") * 2.0
+    row_idx = torch.sort(torch.randperm(N, generator=g, device="cuda")[:m]).values.to(torch.int32)
+    rope = kvb.RopeTable(cfg, N)
+    q = torch.empty(m, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
+    kc = torch.zeros(N, SHAPE.kv_dim, dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros(N, SHAPE.kv_dim, dtype=torch.float16, device="cuda")
+    ws = kvb.workspace(cfg, m)
+    kvb.gather_rmsnorm_qkv(cfg, lws, rope, x_all, row_idx, row_idx, m, q, kc, vc, row_idx, ws)
+    attn = torch.randn(m, SHAPE.q_dim, generator=g, device="cuda").to(torch.bfloat16)
+    x = x_all[row_idx.long()].contiguous()
+    x_in = x.cpu()
+    kvb.mlp_rows(cfg, lws, attn, x, ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    smp = sample_rows(m, 40)
+    ri = row_idx.cpu().numpy()[smp]
+    qr, kr, vr = llama.qkv_rows(s, lw_cpu, np64(x_all.cpu()[ri]), ri)
+    assert_close_bf16(q.cpu()[smp], qr.reshape(len(smp), -1), "q at full size")
+    assert_close_bf16(kc.cpu()[ri], kr.reshape(len(smp), -1), "k at full size (scattered to the rows' cache index)")
+    assert_close_bf16(vc.cpu()[ri], vr.reshape(len(smp), -1), "v at full size")
+    ref = llama.attn_out_mlp(s, lw_cpu, np64(x_in[smp]), np64(attn.cpu()[smp]))
+    e = assert_close_abs(x.cpu()[smp], ref, "x after O-proj + MLP at full size")
+    print("gemm full size", m, e)
+
+
+def test_realign_full_size_sampled_rows(kvb):
+    """All 31 cached layers of the 242 x 512 request (16 GB of chunk caches)."""
+    cfg = kvb.config(SHAPE)
+    L = SHAPE.n_layers - 1
+    g = gen(3)
+    ks = torch.randn(L, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
+    vs = torch.randn(L, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.float16)
+    kd = torch.empty(L, N, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
+    vd = torch.empty(L, N, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.float16, device="cuda")
+    rope = kvb.RopeTable(cfg, N)
+    starts = WL.chunk_starts()
+    kvb.rope_realign(cfg, rope, ks, vs, kd, vd, 0, L, torch.tensor(starts, dtype=torch.int32, device="cuda"), N_CTX)
+    torch.cuda.synchronize()
+    assert torch.equal(vd[:, :N_CTX], vs)
+    smp = np.unique(np.concatenate([[0, 511, 512, N_CTX - 1], np.random.default_rng(4).choice(N_CTX, 60)]))
+    got = kd[:, smp].cpu()
+    # the oracle rotates each sampled row by its own chunk's offset
+    src = np64(ks[:, smp].cpu())
+    want = np.empty_like(src)
+    for j, t in enumerate(smp):
+        c = int(np.searchsorted(starts, t, side="right") - 1)
+        want[:, j:j + 1] = _rot(src[:, j:j + 1], starts[c])
+    assert_close_bf16(got, want, "re-aligned keys at full size")
+
+
+def _rot(k, offset):
+    s = Shape.of(SHAPE, act_bf16=True)
+    c, sn = llama.rope_cos_sin(s, [offset])
+    flat = k.reshape(-1, k.shape[-2], k.shape[-1])
+    r = llama.apply_rope(flat, np.broadcast_to(c, (flat.shape[0], c.shape[1])),
+                         np.broadcast_to(sn, (flat.shape[0], sn.shape[1])))
+    return llama.bf16_round(r.reshape(k.shape))
+
+
+@pytest.fixture(scope="module")
+def headline(kvb):
+    """The benchmark's request: 32 layers, 242 x 512 + 128 tokens, caches from isolated prefill."""
+    cfg = kvb.config(SHAPE)
+    w = workload.device_model(SHAPE, seed=0, device="cuda", draw_on_device=True)
+    model = kvb.Model(w)
+    toks = synth.make_tokens(SHAPE, N, 1).cuda()
+    rope = kvb.RopeTable(cfg, N)
+    ws = kvb.workspace(cfg, N)
+    starts = WL.chunk_starts()
+    kch, vch = workload.chunk_caches(cfg, model, rope, toks[:N_CTX], starts, ws=ws)
+    torch.cuda.synchronize()
+    return dict(cfg=cfg, model=model, toks=toks, rope=rope, ws=ws, starts=starts, kch=kch, vch=vch,
+                dstarts=torch.tensor(starts, dtype=torch.int32, device="cuda"))
+
+
+def _cache():
+    k = torch.empty(SHAPE.n_layers, N, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
+    return k, torch.empty(k.shape, dtype=torch.float16, device="cuda")
+
+
+def test_headline_selective_prefill_properties(kvb, headline):
+    h = headline
+    ck, cv = _cache()
+    fh, sel, t = kvb.selective_prefill(h["cfg"], h["model"], h["rope"], h["kch"], h["vch"], ck, cv, h["toks"],
+                                       h["dstarts"], N_CTX, WL.n_query, WL.r, 1, ws=h["ws"], timings=True)
+    torch.cuda.synchronize()
+    assert kvb.device_status(h["ws"]) == 0
+    k = blend.num_selected(WL.r, N_CTX)
+    assert t["n_selected"] == k and t["n_rows"] == k + WL.n_query
+    s = sel[:k].cpu().numpy()
+    assert len(np.unique(s)) == k and np.all(np.diff(s) > 0) and s[-1] < N_CTX
+    assert torch.isfinite(fh).all()
+    # unselected context rows of every cached layer hold exactly the re-aligned chunk caches
+    kd, vd = _cache()
+    kvb.rope_realign(h["cfg"], h["rope"], h["kch"], h["vch"], kd, vd, 1, SHAPE.n_layers, h["dstarts"], N_CTX)
+    torch.cuda.synchronize()
+    keep = np.ones(N_CTX, dtype=bool)
+    keep[s] = False
+    keep_t = torch.from_numpy(keep).cuda()
+    for l in (1, 2, 15, 31):
+        assert torch.equal(ck[l, :N_CTX][keep_t], kd[l, :N_CTX][keep_t]), l
+        assert torch.equal(cv[l, :N_CTX][keep_t], vd[l, :N_CTX][keep_t]), l
+        # recomputed rows got fresh keys (they differ from the cached ones)
+        assert not torch.equal(ck[l, :N_CTX][~keep_t], kd[l, :N_CTX][~keep_t]), l
+    # a second run gives the same bits
+    ck2, cv2 = _cache()
+    fh2, sel2, _ = kvb.selective_prefill(h["cfg"], h["model"], h["rope"], h["kch"], h["vch"], ck2, cv2, h["toks"],
+                                         h["dstarts"], N_CTX, WL.n_query, WL.r, 1, ws=h["ws"])
+    torch.cuda.synchronize()
+    assert torch.equal(fh, fh2) and torch.equal(sel[:k], sel2[:k]) and torch.equal(ck, ck2)
+
+
+def test_headline_selection_matches_step_api_composition(kvb, headline):
+    """Rebuild the check layer from the public step entry points (layer 0 over all rows,
+    fresh layer-1 keys of every context row, deviation against the re-aligned cache,
+    top-k) and require the whole-path call to have chosen exactly the same rows, and
+    those rows to be a top-k of the deviation (every chosen value >= every other)."""
+    h = headline
+    cfg = h["cfg"]
+    ws = h["ws"]
+    ck, cv = _cache()
+    _, sel, _ = kvb.selective_prefill(cfg, h["model"], h["rope"], h["kch"], h["vch"], ck, cv, h["toks"],
+                                      h["dstarts"], N_CTX, WL.n_query, WL.r, 1, ws=ws)
+    torch.cuda.synchronize()
+    k = blend.num_selected(WL.r, N_CTX)
+    sel_path = sel[:k].clone()
+    del ck, cv
+    W = h["model"].weights
+    x = W["embed"][h["toks"].long()].float().contiguous()          # layer-0 input: embedding rows
+    ident = torch.arange(N, dtype=torch.int32, device="cuda")
+    q = torch.empty(N, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
+    k0 = torch.empty(N, SHAPE.kv_dim, dtype=torch.bfloat16, device="cuda")
+    v0 = torch.empty(N, SHAPE.kv_dim, dtype=torch.float16, device="cuda")
+    lw0 = kvb.layer_struct(W["layers"][0])
+    kvb.gather_rmsnorm_qkv(cfg, lw0, h["rope"], x, None, ident, N, q, k0, v0, None, ws)
+    attn = torch.empty(N, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
+    kvb.sparse_query_attn(cfg, q, ident, None, k0.view(N, SHAPE.n_kv_heads, SHAPE.head_dim),
+                          v0.view(N, SHAPE.n_kv_heads, SHAPE.head_dim), attn, ws)
+    kvb.mlp_rows(cfg, lw0, attn, x, ws)                              # x <- layer-0 output
+    lw1 = kvb.layer_struct(W["layers"][1])
+    qf = torch.empty(N_CTX, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
+    kf = torch.empty(N_CTX, SHAPE.kv_dim, dtype=torch.bfloat16, device="cuda")
+    vf = torch.empty(N_CTX, SHAPE.kv_dim, dtype=torch.float16, device="cuda")
+    kvb.gather_rmsnorm_qkv(cfg, lw1, h["rope"], x, None, ident[:N_CTX], N_CTX, qf, kf, vf, None, ws)
+    kd = torch.empty(2, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
+    vd = torch.empty(kd.shape, dtype=torch.float16, device="cuda")
+    kvb.rope_realign(cfg, h["rope"], h["kch"], h["vch"], kd, vd, 1, 2, h["dstarts"], N_CTX)
+    sel2, dev = kvb.hkvd_select(kf, kd[1].reshape(N_CTX, -1), k)
+    torch.cuda.synchronize()
+    assert kvb.device_status(ws) == 0
+    assert torch.equal(sel_path, sel2)
+    d = dev.cpu().numpy()
+    chosen = np.zeros(N_CTX, dtype=bool)
+    chosen[sel2.cpu().numpy()] = True
+    assert d[chosen].min() >= d[~chosen].max()
+
+
+def test_headline_full_ratio_equals_dense_prefill(kvb, headline):
+    h = headline
+    ck, cv = _cache()
+    fh, sel, _ = kvb.selective_prefill(h["cfg"], h["model"], h["rope"], h["kch"], h["vch"], ck, cv, h["toks"],
+                                       h["dstarts"], N_CTX, WL.n_query, 1.0, 1, ws=h["ws"])
+    ck2, cv2 = _cache()
+    fh2, _ = kvb.full_prefill(h["cfg"], h["model"], h["rope"], ck2, cv2, h["toks"], n_out=WL.n_query, ws=h["ws"])
+    torch.cuda.synchronize()
+    assert torch.equal(fh, fh2) and torch.equal(ck, ck2) and torch.equal(cv, cv2)
+    assert torch.isfinite(fh).all()
