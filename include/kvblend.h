@@ -293,6 +293,36 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
                                  float* final_hidden, int32_t* sel_out,
                                  kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
 
+/* The same prefill with the chunk caches in pinned HOST memory, ingested layer by layer
+ * while the model computes (Sec. 3.4: KV caches are transferred to the GPU, merged and
+ * position-adjusted layer by layer, overlapped with the recompute through CUDA streams).
+ * For every cached layer l the library copies layer l of k_chunks_host / v_chunks_host
+ * into one of two device staging slots on `copy_stream`, merges and re-aligns it into
+ * `cache` there, and makes `stream` wait for that layer only just before it first reads
+ * or writes cache layer l; layer 0 (and every layer before check_layer) needs no cache, so
+ * the ingest runs under its compute.  k_chunks_host / v_chunks_host: pinned host memory
+ * (cudaHostAlloc or registered), [n_layers][n_ctx][Hkv][D], K bf16 / V fp16.  copy_stream:
+ * a stream other than `stream`.  Workspace: kvb_workspace_size_pipelined(cfg, n_ctx +
+ * n_query, n_ctx) bytes (the staging slots follow the regular layout).  All other
+ * arguments and results as kvb_selective_prefill; realign_ms in `t` is 0 here because the
+ * merge runs on copy_stream.  Errors: as kvb_selective_prefill, INVALID_ARG if the chunk
+ * caches are not pinned host memory or copy_stream == stream. */
+kvb_status kvb_selective_prefill_host(const kvb_config* cfg, const kvb_model* model,
+                                      const kvb_rope_table* rope,
+                                      const uint16_t* k_chunks_host, const uint16_t* v_chunks_host,
+                                      kvb_kv_cache* cache,
+                                      const int32_t* token_ids, const int32_t* chunk_start,
+                                      int32_t n_chunks, int64_t n_ctx, int64_t n_query,
+                                      float r, int32_t check_layer,
+                                      const int32_t* forced_sel, int64_t forced_k,
+                                      float* final_hidden, int32_t* sel_out,
+                                      kvb_timings* t, void* ws, size_t ws_bytes,
+                                      void* stream, void* copy_stream);
+
+/* Workspace bytes for kvb_selective_prefill_host: kvb_workspace_size(cfg, n_rows) plus two
+ * staging slots of one layer of chunk K and V for n_ctx rows. */
+kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, int64_t n_ctx, size_t* bytes);
+
 /* Dense causal prefill of n rows through every layer (the r = 1 comparator, Sec. 4;
  * also the per-chunk isolated prefill that produces chunk caches):
  *   row t attends cache rows [kv_lo[t], t] (kv_lo NULL = 0) with RoPE at rope_pos[t]

@@ -582,12 +582,25 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
     return KVB_OK;
 }
 
-kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
+}  // extern "C"
+
+// Bytes of the two staging slots the pipelined (host-resident chunk caches) prefill needs:
+// one layer of chunk K and V per slot.
+static size_t staging_bytes(const kvb_config* c, int64_t n_ctx) {
+    const size_t layer = (size_t)(n_ctx > 0 ? n_ctx : 0) * (size_t)c->n_kv_heads * c->head_dim * 2;
+    return 2 * 2 * ((layer + 255) / 256 * 256);
+}
+
+// The selective prefill.  With host_src, k_chunks / v_chunks are pinned host memory:
+// each cached layer is copied into one of two device staging slots on copy_st and merged
+// + re-aligned there, and the compute stream waits for layer l's event just before it
+// first reads or writes cache layer l (the per-layer overlap of Sec. 3.4).
+static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
                                  const uint16_t* k_chunks, const uint16_t* v_chunks, kvb_kv_cache* cache,
                                  const int32_t* token_ids, const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
                                  int64_t n_query, float r, int32_t check_layer_idx, const int32_t* forced_sel,
                                  int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
-                                 size_t ws_bytes, void* stream) {
+                                 size_t ws_bytes, void* stream, bool host_src, void* copy_stream) {
     g_err[0] = 0;
     KVB_TRY(check_cfg(cfg));
     KVB_TRY(check_model(cfg, model));
@@ -612,8 +625,21 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
         KVB_TRY(check_ptr(v_chunks, "v_chunks"));
         KVB_TRY(check_ptr(chunk_start, "chunk_start"));
         if (n_chunks < 1) return fail(KVB_ERR_INVALID_ARG, "selective prefill: n_chunks < 1");
+        if (host_src) {
+            for (const void* hp : {static_cast<const void*>(k_chunks), static_cast<const void*>(v_chunks)}) {
+                cudaPointerAttributes a;
+                if (cudaPointerGetAttributes(&a, hp) != cudaSuccess || a.type != cudaMemoryTypeHost) {
+                    cudaGetLastError();
+                    return fail(KVB_ERR_INVALID_ARG, "pipelined prefill: chunk caches must be pinned host memory");
+                }
+            }
+        }
     }
     Workspace w;
+    const size_t ws_main = workspace_layout(cfg, N, nullptr, &w);
+    const size_t ws_need = ws_main + (host_src ? staging_bytes(cfg, n_ctx) : 0);
+    if (ws_bytes < ws_need)
+        return fail(KVB_ERR_WORKSPACE, "workspace %zu bytes < %zu needed", ws_bytes, ws_need);
     KVB_TRY(carve(cfg, N, ws, ws_bytes, &w));
     Ctx c = make_ctx(cfg, rope, w, stream);
     Prof prof;
@@ -628,10 +654,47 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
     tm.start(t != nullptr, c.st);
     const int lc = dense_all ? L : check_layer_idx;
     // 1. merge + re-align the chunk caches of the layers that will be read as cached
-    if (lc < L && n_ctx > 0)
+    struct Events {
+        std::vector<cudaEvent_t> ev;
+        ~Events() {
+            for (auto e : ev)
+                if (e) cudaEventDestroy(e);
+        }
+    } ready;
+    ready.ev.assign((size_t)L, nullptr);
+    if (lc < L && n_ctx > 0 && !host_src) {
         KVB_TRY(launch_realign(rope->cos, rope->sin, c.D, c.Hkv, k_chunks + (int64_t)lc * n_ctx * kvd,
                                v_chunks + (int64_t)lc * n_ctx * kvd, n_ctx * kvd, kc(lc), vc(lc), rows_c * kvd,
                                L - lc, chunk_start, n_chunks, n_ctx, c.st));
+    } else if (lc < L && n_ctx > 0) {
+        cudaStream_t cs = static_cast<cudaStream_t>(copy_stream);
+        cudaEvent_t go = nullptr;
+        KVB_TRY(cuda_ok(cudaEventCreateWithFlags(&go, cudaEventDisableTiming), "pipelined prefill: event"));
+        kvb_status st = cuda_ok(cudaEventRecord(go, c.st), "pipelined prefill: record");
+        if (st == KVB_OK) st = cuda_ok(cudaStreamWaitEvent(cs, go, 0), "pipelined prefill: wait");
+        cudaEventDestroy(go);
+        KVB_TRY(st);
+        const size_t layer_elems = (size_t)n_ctx * kvd;
+        const size_t slot = staging_bytes(cfg, n_ctx) / 4;   // bytes of one K (or V) slot
+        char* stage = static_cast<char*>(ws) + ws_main;
+        for (int l = lc; l < L; ++l) {
+            const int sl = (l - lc) & 1;
+            uint16_t* sk = reinterpret_cast<uint16_t*>(stage + (size_t)(2 * sl) * slot);
+            uint16_t* sv = reinterpret_cast<uint16_t*>(stage + (size_t)(2 * sl + 1) * slot);
+            KVB_TRY(cuda_ok(cudaMemcpyAsync(sk, k_chunks + (size_t)l * layer_elems, layer_elems * 2,
+                                            cudaMemcpyHostToDevice, cs), "pipelined prefill: K copy"));
+            KVB_TRY(cuda_ok(cudaMemcpyAsync(sv, v_chunks + (size_t)l * layer_elems, layer_elems * 2,
+                                            cudaMemcpyHostToDevice, cs), "pipelined prefill: V copy"));
+            KVB_TRY(launch_realign(rope->cos, rope->sin, c.D, c.Hkv, sk, sv, (int64_t)layer_elems, kc(l), vc(l),
+                                   rows_c * kvd, 1, chunk_start, n_chunks, n_ctx, cs));
+            KVB_TRY(cuda_ok(cudaEventCreateWithFlags(&ready.ev[l], cudaEventDisableTiming), "pipelined prefill: event"));
+            KVB_TRY(cuda_ok(cudaEventRecord(ready.ev[l], cs), "pipelined prefill: record"));
+        }
+    }
+    auto wait_layer = [&](int l) -> kvb_status {
+        if (l < 0 || l >= L || !ready.ev[l]) return KVB_OK;
+        return cuda_ok(cudaStreamWaitEvent(c.st, ready.ev[l], 0), "pipelined prefill: layer wait");
+    };
     tm.mark();
     // 2. dense layers (layer 0 at least): every row, causal
     KVB_TRY(launch_iota(w.ident, N, 0, c.st));
@@ -654,6 +717,7 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
                 p.k_out = w.k_fresh; p.rope_pos = w.ident; p.cos_t = rope->cos; p.sin_t = rope->sin;
                 p.status = w.status;
                 KVB_TRY(gemm(c, p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr));
+                KVB_TRY(wait_layer(lc));
                 KVB_TRY(launch_hkvd(w.k_fresh, kvd, kc(lc), kvd, n_ctx, (int)kvd, k, w.sel, w.dev, w.topk, c.st));
             }
             sel = w.sel;
@@ -665,8 +729,10 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
             KVB_TRY(cuda_ok(cudaMemcpyAsync(sel_out, sel, (size_t)k * 4, cudaMemcpyDeviceToDevice, c.st), "sel copy"));
         tm.mark();
         // 4. selective layers over the recomputed rows
-        for (int l = lc; l < L; ++l)
+        for (int l = lc; l < L; ++l) {
+            KVB_TRY(wait_layer(l));
             KVB_TRY(layer(c, &model->layers[l], w.x_sel, m, w.rows, w.rows, nullptr, kc(l), vc(l), N));
+        }
         x_final = w.x_sel;
     } else {
         if (sel_out && n_ctx > 0) KVB_TRY(launch_iota(sel_out, n_ctx, 0, c.st));
@@ -692,6 +758,42 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
         t->n_rows = m;
         fill_kernel_times(prof, t, launch_count() - launches0);
     }
+    return KVB_OK;
+}
+
+
+extern "C" {
+
+kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
+                                 const uint16_t* k_chunks, const uint16_t* v_chunks, kvb_kv_cache* cache,
+                                 const int32_t* token_ids, const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
+                                 int64_t n_query, float r, int32_t check_layer, const int32_t* forced_sel,
+                                 int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
+                                 size_t ws_bytes, void* stream) {
+    return selective_impl(cfg, model, rope, k_chunks, v_chunks, cache, token_ids, chunk_start, n_chunks, n_ctx,
+                          n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, ws, ws_bytes,
+                          stream, false, nullptr);
+}
+
+kvb_status kvb_selective_prefill_host(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
+                                      const uint16_t* k_chunks_host, const uint16_t* v_chunks_host,
+                                      kvb_kv_cache* cache, const int32_t* token_ids, const int32_t* chunk_start,
+                                      int32_t n_chunks, int64_t n_ctx, int64_t n_query, float r,
+                                      int32_t check_layer, const int32_t* forced_sel, int64_t forced_k,
+                                      float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
+                                      size_t ws_bytes, void* stream, void* copy_stream) {
+    if (copy_stream == stream) return fail(KVB_ERR_INVALID_ARG, "pipelined prefill: copy_stream must differ from stream");
+    return selective_impl(cfg, model, rope, k_chunks_host, v_chunks_host, cache, token_ids, chunk_start, n_chunks,
+                          n_ctx, n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, ws, ws_bytes,
+                          stream, true, copy_stream);
+}
+
+kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, int64_t n_ctx, size_t* bytes) {
+    g_err[0] = 0;
+    KVB_TRY(check_cfg(cfg));
+    if (!bytes || n_rows < 0 || n_ctx < 0) return fail(KVB_ERR_INVALID_ARG, "workspace size: bad arguments");
+    Workspace w;
+    *bytes = workspace_layout(cfg, n_rows, nullptr, &w) + staging_bytes(cfg, n_ctx);
     return KVB_OK;
 }
 

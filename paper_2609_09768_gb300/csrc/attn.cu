@@ -8,14 +8,20 @@
 // of the selective layers, the dense causal prefill and the block-diagonal
 // per-chunk prefill.
 //
+// Both A operands live in tensor memory, so each MMA reads only its K or V tile
+// from shared memory: with A and B both in shared memory an M128 x N128 step
+// needs the whole shared-memory bandwidth on its own, before the TMA writes.
+// TMEM columns: S double buffer [0, 256), O [256, 384), Q [384, 448), P [448, 512).
+//
 // Pipeline per key tile j (128 keys):
-//   TMA warp   : K_j, V_j into 2-deep rings (128-byte swizzle)
-//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=128, K=16 steps);
-//                after the softmax of tile j-1, O += P_{j-1} V_{j-1} (V as an
-//                MN-major operand, O accumulated in TMEM)
-//   4 softmax warps (thread = row): read S_j from TMEM, mask, online softmax with
-//                a lazily updated running max (O is rescaled only when the max
-//                grows by more than 2^8), write P_j to swizzled smem.
+//   TMA warp   : K_j, V_j into 3-deep rings (128-byte swizzle)
+//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=128, K=16 steps,
+//                A = Q from TMEM); after the softmax of tile j-1,
+//                O += P_{j-1} V_{j-1} (A = P from TMEM, V an MN-major operand)
+//   4 softmax warps (thread = row): load the row's Q into TMEM once; per tile
+//                read S_j from TMEM, mask, online softmax with a lazily updated
+//                running max (O is rescaled only when the max grows by more than
+//                2^8), write P_j into its TMEM columns once P.V_{j-1} is done.
 // Lazy rescaling keeps the result exact: every term uses the same reference max
 // as the running sum it is divided by.
 // Precision: Q.K^T runs on bf16 operands; P.V runs on fp16 operands - the
@@ -32,43 +38,41 @@ namespace {
 
 constexpr int THREADS = 192;
 constexpr int KT_ROWS = 128;                 // keys per tile
+constexpr int STAGES = 3;                    // K and V ring depth
 constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t COL_S = 0, COL_O = 256, COL_Q = 384, COL_P = 448;
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
 
 template <int D>
 struct Smem {
     static constexpr int CHUNK = 128 * 128;              // 128 rows x 128 bytes
-    static constexpr int Q_BYTES = (D / 64) * CHUNK;
     static constexpr int KV_BYTES = (D / 64) * CHUNK;    // one K or V tile
-    static constexpr int P_BYTES = 2 * CHUNK;            // 128 rows x 128 keys bf16
-    static constexpr int OFF_Q = 0;
-    static constexpr int OFF_K = OFF_Q + Q_BYTES;
-    static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
-    static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
-    static constexpr int OFF_BAR = OFF_P + P_BYTES;
+    static constexpr int OFF_K = 0;
+    static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
+    static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
     static constexpr int TOTAL = OFF_BAR + 256 + 1024;
 };
 
 template <int D>
 __global__ void __launch_bounds__(THREADS, 1)
-attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap tmK,
             const __grid_constant__ CUtensorMap tmV, const AttnParams p, int num_blocks) {
     using S = Smem<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
-    uint64_t* q_full = bars + 0;
-    uint64_t* k_full = bars + 1;     // [2]
-    uint64_t* k_empty = bars + 3;    // [2]
-    uint64_t* v_full = bars + 5;     // [2]
-    uint64_t* v_empty = bars + 7;    // [2]
-    uint64_t* s_full = bars + 9;     // [2]
-    uint64_t* s_free = bars + 11;    // [2]
-    uint64_t* p_full = bars + 13;
-    uint64_t* pv_done = bars + 14;
-    uint64_t* drain = bars + 15;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+    uint64_t* q_ready = bars + 0;                // Q rows stored into TMEM (4 warps)
+    uint64_t* k_full = bars + 1;                 // [STAGES]
+    uint64_t* k_empty = k_full + STAGES;         // [STAGES]
+    uint64_t* v_full = k_empty + STAGES;         // [STAGES]
+    uint64_t* v_empty = v_full + STAGES;         // [STAGES]
+    uint64_t* s_full = v_empty + STAGES;         // [2]
+    uint64_t* s_free = s_full + 2;               // [2]
+    uint64_t* p_full = s_free + 2;
+    uint64_t* pv_done = p_full + 1;
+    uint64_t* drain = pv_done + 1;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* red = reinterpret_cast<int*>(tmem_slot + 2);   // lo_min, hi_max, hi_min, lo_max
 
@@ -80,12 +84,12 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     const int64_t r0 = (int64_t)blk * RPB;
 
     if (threadIdx.x == 0) {
-        mbar_init(q_full, 1);
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(&k_full[b], 1); mbar_init(&k_empty[b], 1);
-            mbar_init(&v_full[b], 1); mbar_init(&v_empty[b], 1);
-            mbar_init(&s_full[b], 1); mbar_init(&s_free[b], 4);
+        mbar_init(q_ready, 4);
+        for (int st = 0; st < STAGES; ++st) {
+            mbar_init(&k_full[st], 1); mbar_init(&k_empty[st], 1);
+            mbar_init(&v_full[st], 1); mbar_init(&v_empty[st], 1);
         }
+        for (int b = 0; b < 2; ++b) { mbar_init(&s_full[b], 1); mbar_init(&s_free[b], 4); }
         mbar_init(p_full, 4);
         mbar_init(pv_done, 1);
         mbar_init(drain, 1);
@@ -111,7 +115,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         atomicMin(&red[2], hi);
         atomicMax(&red[3], lo);
     }
-    if (warp == 0 && lane == 0) { prefetch_tmap(&tmQ); prefetch_tmap(&tmK); prefetch_tmap(&tmV); }
+    if (warp == 0 && lane == 0) { prefetch_tmap(&tmK); prefetch_tmap(&tmV); }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -120,43 +124,40 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     const int t_begin = lo_min / KT_ROWS;
     const int n_tiles = hi_max < 0 ? 0 : hi_max / KT_ROWS + 1 - t_begin;
 
-    uint8_t* sQ = smem + S::OFF_Q;
     uint8_t* sK = smem + S::OFF_K;
     uint8_t* sV = smem + S::OFF_V;
-    uint8_t* sP = smem + S::OFF_P;
 
     if (warp == 0) {
         if (lane == 0 && n_tiles > 0) {
             // ------------------------------------------------ TMA producer
-            mbar_expect_tx(q_full, S::Q_BYTES);
-#pragma unroll
-            for (int c = 0; c < D / 64; ++c) tma_load_3d(sQ + c * S::CHUNK, &tmQ, q_full, c * 64, g * G, (int)r0);
-            int issued_k = 0, issued_v = 0;
+            int issued = 0;
             for (int j = 0; j < n_tiles; ++j) {
-                const int b = j & 1;
-                const uint32_t ph = (j >> 1) & 1;
+                const int st = j % STAGES;
+                const uint32_t ph = (uint32_t)(j / STAGES) & 1;
                 const int y = (t_begin + j) * KT_ROWS;
-                if (!mbar_wait(&k_empty[b], ph ^ 1, abort_flag, p.status)) break;
-                mbar_expect_tx(&k_full[b], S::KV_BYTES);
+                if (!mbar_wait(&k_empty[st], ph ^ 1, abort_flag, p.status)) break;
+                mbar_expect_tx(&k_full[st], S::KV_BYTES);
 #pragma unroll
                 for (int c = 0; c < D / 64; ++c)
-                    tma_load_2d(sK + b * S::KV_BYTES + c * S::CHUNK, &tmK, &k_full[b], g * D + c * 64, y);
-                issued_k = j + 1;
-                if (!mbar_wait(&v_empty[b], ph ^ 1, abort_flag, p.status)) break;
-                mbar_expect_tx(&v_full[b], S::KV_BYTES);
+                    tma_load_2d(sK + st * S::KV_BYTES + c * S::CHUNK, &tmK, &k_full[st], g * D + c * 64, y);
+                if (!mbar_wait(&v_empty[st], ph ^ 1, abort_flag, p.status)) { issued = -(j + 1); break; }
+                mbar_expect_tx(&v_full[st], S::KV_BYTES);
 #pragma unroll
                 for (int c = 0; c < D / 64; ++c)
-                    tma_load_2d(sV + b * S::KV_BYTES + c * S::CHUNK, &tmV, &v_full[b], g * D + c * 64, y);
-                issued_v = j + 1;
+                    tma_load_2d(sV + st * S::KV_BYTES + c * S::CHUNK, &tmV, &v_full[st], g * D + c * 64, y);
+                issued = j + 1;
             }
             // on the abort path, let the loads already issued land before exiting
             if (*abort_flag) {
+                const int nk = issued < 0 ? -issued : issued;      // K tiles issued
+                const int nv = issued < 0 ? -issued - 1 : issued;  // V tiles issued
                 const uint64_t t0 = globaltimer();
-                for (int j = (issued_k > 2 ? issued_k - 2 : 0); j < issued_k; ++j)
-                    while (!mbar_try_wait(&k_full[j & 1], (j >> 1) & 1) && globaltimer() - t0 < 1000000ull) {}
-                for (int j = (issued_v > 2 ? issued_v - 2 : 0); j < issued_v; ++j)
-                    while (!mbar_try_wait(&v_full[j & 1], (j >> 1) & 1) && globaltimer() - t0 < 1000000ull) {}
-                while (!mbar_try_wait(q_full, 0) && globaltimer() - t0 < 1000000ull) {}
+                for (int j = (nk > STAGES ? nk - STAGES : 0); j < nk; ++j)
+                    while (!mbar_try_wait(&k_full[j % STAGES], (uint32_t)(j / STAGES) & 1) &&
+                           globaltimer() - t0 < 1000000ull) {}
+                for (int j = (nv > STAGES ? nv - STAGES : 0); j < nv; ++j)
+                    while (!mbar_try_wait(&v_full[j % STAGES], (uint32_t)(j / STAGES) & 1) &&
+                           globaltimer() - t0 < 1000000ull) {}
             }
         }
     } else if (warp == 1) {
@@ -164,38 +165,38 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
             // ------------------------------------------------ MMA issuer
             constexpr uint32_t IDESC_S = idesc_bf16(128, KT_ROWS, false);
             constexpr uint32_t IDESC_O = idesc_f16kind(128, D, true, false);   // fp16 P and V
-            const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(sK), v0 = smem_u32(sV), p0 = smem_u32(sP);
-            bool ok = mbar_wait(q_full, 0, abort_flag, p.status);
+            const uint32_t k0 = smem_u32(sK), v0 = smem_u32(sV);
+            bool ok = mbar_wait(q_ready, 0, abort_flag, p.status);
             tc_fence_after();
             for (int j = 0; ok && j <= n_tiles; ++j) {
                 if (j < n_tiles) {
-                    const int b = j & 1;
-                    if (!mbar_wait(&k_full[b], (j >> 1) & 1, abort_flag, p.status)) break;
+                    const int b = j & 1, st = j % STAGES;
+                    if (!mbar_wait(&k_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status)) break;
                     if (j >= 2 && !mbar_wait(&s_free[b], ((j - 2) >> 1) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
-                    const uint32_t kb = k0 + b * S::KV_BYTES;
+                    const uint32_t kb = k0 + st * S::KV_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * S::CHUNK + (kk & 3) * 32;
-                        mma_bf16_ss(tmem_base + b * KT_ROWS, sdesc_sw128(q0 + off, 16, 1024),
-                                    sdesc_sw128(kb + off, 16, 1024), IDESC_S, kk > 0);
+                        // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
+                        mma_f16_ts(tmem_base + COL_S + b * KT_ROWS, tmem_base + COL_Q + kk * 8,
+                                   sdesc_sw128(kb + (kk >> 2) * S::CHUNK + (kk & 3) * 32, 16, 1024), IDESC_S, kk > 0);
                     }
-                    mma_commit(&k_empty[b]);
+                    mma_commit(&k_empty[st]);
                     mma_commit(&s_full[b]);
                 }
                 if (j >= 1) {
-                    const int i = j - 1, bi = i & 1;
+                    const int i = j - 1, st = i % STAGES;
                     if (!mbar_wait(p_full, i & 1, abort_flag, p.status)) break;
-                    if (!mbar_wait(&v_full[bi], (i >> 1) & 1, abort_flag, p.status)) break;
+                    if (!mbar_wait(&v_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
-                    const uint32_t vb = v0 + bi * S::KV_BYTES;
+                    const uint32_t vb = v0 + st * S::KV_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < KT_ROWS / 16; ++kk) {
-                        const uint32_t offp = (kk >> 2) * S::CHUNK + (kk & 3) * 32;
-                        mma_bf16_ss(tmem_base + 2 * KT_ROWS, sdesc_sw128(p0 + offp, 16, 1024),
-                                    sdesc_sw128(vb + kk * 16 * 128, S::CHUNK, 1024), IDESC_O, (i > 0) || (kk > 0));
+                        // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
+                        mma_f16_ts(tmem_base + COL_O, tmem_base + COL_P + kk * 8,
+                                   sdesc_sw128(vb + kk * 16 * 128, S::CHUNK, 1024), IDESC_O, (i > 0) || (kk > 0));
                     }
-                    mma_commit(&v_empty[bi]);
+                    mma_commit(&v_empty[st]);
                     mma_commit(pv_done);
                 }
             }
@@ -209,6 +210,27 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         const uint32_t lane_addr = (quarter * 32u) << 16;
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
+        {
+            // this row's query into TMEM columns [COL_Q, COL_Q + D/2): bf16 pairs, lane = row
+            uint32_t qv[D / 2];
+            if (valid) {
+                const uint4* src = reinterpret_cast<const uint4*>(q + row * (int64_t)(p.Hq * D) + (int64_t)head * D);
+#pragma unroll
+                for (int c = 0; c < D / 8; ++c) {
+                    const uint4 u = __ldg(src + c);
+                    qv[4 * c] = u.x; qv[4 * c + 1] = u.y; qv[4 * c + 2] = u.z; qv[4 * c + 3] = u.w;
+                }
+            } else {
+#pragma unroll
+                for (int c = 0; c < D / 2; ++c) qv[c] = 0u;
+            }
+#pragma unroll
+            for (int c = 0; c < D / 64; ++c) tmem_st32(tmem_base + lane_addr + COL_Q + c * 32, qv + c * 32);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(q_ready);
+        }
         for (int j = 0; j < n_tiles; ++j) {
             const int b = j & 1;
             if (!mbar_wait_warp(&s_full[b], (j >> 1) & 1, abort_flag, p.status)) { ok = false; break; }
@@ -261,7 +283,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
                 if (!mbar_wait_warp(pv_done, (j - 1) & 1, abort_flag, p.status)) { ok = false; break; }
                 tc_fence_after();
                 if (__any_sync(0xffffffffu, resc)) {
-                    const uint32_t oaddr = tmem_base + lane_addr + 2 * KT_ROWS;
+                    const uint32_t oaddr = tmem_base + lane_addr + COL_O;
 #pragma unroll 1
                     for (int c = 0; c < D / 32; ++c) {
                         uint32_t o[32];
@@ -274,21 +296,17 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
                     tmem_st_wait();
                 }
             }
-            // P row L into the 128-byte-swizzled K-major operand layout
-#pragma unroll
-            for (int u = 0; u < KT_ROWS / 8; ++u) {
-                const int chunk = u >> 3, uu = u & 7;
-                uint8_t* dst = sP + chunk * S::CHUNK + (L >> 3) * 1024 + (L & 7) * 128 + ((uu ^ (L & 7)) << 4);
-                *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-            }
-            fence_async_smem();
+            // P row L (fp16 pairs) into its TMEM columns; P.V_{j-1} has finished reading them
+            tmem_st32(tmem_base + lane_addr + COL_P, pk);
+            tmem_st32(tmem_base + lane_addr + COL_P + 32, pk + 32);
+            tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(p_full);
         }
         if (ok && mbar_wait_warp(pv_done, (n_tiles - 1) & 1, abort_flag, p.status)) {
             tc_fence_after();
-            const uint32_t oaddr = tmem_base + lane_addr + 2 * KT_ROWS;
+            const uint32_t oaddr = tmem_base + lane_addr + COL_O;
             const float inv = (l_run > 0.f) ? 1.f / l_run : 0.f;
             uint16_t* dst = p.out + row * (int64_t)(p.Hq * D) + (int64_t)head * D;
 #pragma unroll 1
@@ -320,7 +338,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
 }
 
 template <int D>
-kvb_status run(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v, const AttnParams& p, int nb,
+kvb_status run(const uint16_t* q, const CUtensorMap& k, const CUtensorMap& v, const AttnParams& p, int nb,
                cudaStream_t st) {
     static bool attr_set = false;
     auto kern = attn_kernel<D>;
@@ -345,17 +363,15 @@ kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k
     if (p.Hkv <= 0 || p.Hq % p.Hkv || 128 % (p.Hq / p.Hkv))
         return fail(KVB_ERR_UNSUPPORTED, "attention: Hq/Hkv must divide 128");
     const int G = p.Hq / p.Hkv, RPB = 128 / G;
-    CUtensorMap tq, tk, tv;
-    kvb_status s = make_tmap_3d(&tq, q, (uint64_t)p.D, (uint64_t)p.Hq, (uint64_t)p.m, 64, (uint32_t)G, (uint32_t)RPB);
-    if (s != KVB_OK) return s;
+    CUtensorMap tk, tv;
     const uint64_t kvd = (uint64_t)p.Hkv * p.D;
-    s = make_tmap_2d(&tk, k_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
+    kvb_status s = make_tmap_2d(&tk, k_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS);
     if (s != KVB_OK) return s;
     s = make_tmap_2d(&tv, v_cache, kvd, (uint64_t)p.n_kv, kvd, 64, KT_ROWS, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
     if (s != KVB_OK) return s;
     const int64_t nb = (p.m + RPB - 1) / RPB;
     if (nb * p.Hkv > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "attention: too many rows");
-    return p.D == 128 ? run<128>(tq, tk, tv, p, (int)nb, st) : run<64>(tq, tk, tv, p, (int)nb, st);
+    return p.D == 128 ? run<128>(q, tk, tv, p, (int)nb, st) : run<64>(q, tk, tv, p, (int)nb, st);
 }
 
 }  // namespace kvb

@@ -81,22 +81,35 @@ KVB_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// try_wait that lets the hardware suspend the thread until the phase completes or
+// `hint_ns` elapses, so waiting warps do not take issue slots from working ones.
+KVB_DEV bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait until the phase with the given parity has completed.  Gives up after
-// kWaitLimitNs (or as soon as another thread of the CTA has given up, signalled
+// limit_ns (or as soon as another thread of the CTA has given up, signalled
 // through *abort), records KVB_ERR_TIMEOUT and returns false.
 KVB_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* status,
                        uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 63u) == 0) {
-            if (*abort) return false;
-            if (globaltimer() - t0 > limit_ns) {
-                *abort = 1;
-                set_status(status, KVB_ERR_TIMEOUT);
-                return false;
-            }
+    const uint32_t hint = limit_ns < 1000000ull ? (uint32_t)(limit_ns / 4 + 1) : 250000u;
+    for (;;) {
+        if (mbar_try_wait_sleep(bar, parity, hint)) return true;
+        if (*abort) return false;
+        if (globaltimer() - t0 > limit_ns) {
+            *abort = 1;
+            set_status(status, KVB_ERR_TIMEOUT);
+            return false;
         }
     }
 }
@@ -152,6 +165,16 @@ KVB_DEV void mma_bf16_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// D[tmem] (+)= A[tmem] * B[smem desc]^T: A (M x K, 16-bit, two elements per 32-bit
+// column, lane = row) read from tensor memory.
+KVB_DEV void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 // Arrive on an mbarrier once all tcgen05 operations issued so far by this thread complete.

@@ -88,6 +88,10 @@ _SIGS = {
     "kvb_selective_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), c_vp, c_vp, P(KVCache), c_vp,
                                       c_vp, c_i32, c_i64, c_i64, c_f32, c_i32, c_vp, c_i64, c_vp, c_vp, P(Timings),
                                       c_vp, c_sz, c_vp]),
+    "kvb_selective_prefill_host": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), c_vp, c_vp, P(KVCache),
+                                           c_vp, c_vp, c_i32, c_i64, c_i64, c_f32, c_i32, c_vp, c_i64, c_vp, c_vp,
+                                           P(Timings), c_vp, c_sz, c_vp, c_vp]),
+    "kvb_workspace_size_pipelined": (c_i32, [P(Config), c_i64, c_i64, P(c_sz)]),
     "kvb_full_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), P(KVCache), c_vp, c_i64, c_vp, c_vp,
                                  c_vp, c_i64, P(Timings), c_vp, c_sz, c_vp]),
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
@@ -305,6 +309,48 @@ def selective_prefill(cfg: Config, model: Model, rope: RopeTable, k_chunks, v_ch
           _ptr(forced_sel, torch.int32, "forced_sel"), forced_sel.numel() if forced_sel is not None else 0,
           _ptr(final_hidden, torch.float32, "final_hidden"), _ptr(sel_out, torch.int32, "sel_out"),
           C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream())
+    return final_hidden[:n_query], sel_out, (t.as_dict() if timings else None)
+
+
+def workspace_size_pipelined(cfg: Config, n_rows: int, n_ctx: int) -> int:
+    n = c_sz(0)
+    _call("kvb_workspace_size_pipelined", C.byref(cfg), n_rows, n_ctx, C.byref(n))
+    return n.value
+
+
+def _host_ptr(t: torch.Tensor, dtype, name: str) -> int:
+    if t.is_cuda or not t.is_pinned():
+        raise ValueError(f"{name} must be a pinned host tensor")
+    if t.dtype != dtype or not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous {dtype}")
+    return t.data_ptr()
+
+
+def selective_prefill_host(cfg: Config, model: Model, rope: RopeTable, k_chunks_host, v_chunks_host, cache_k, cache_v,
+                           token_ids, chunk_start: torch.Tensor, n_ctx: int, n_query: int, r: float,
+                           check_layer: int = 1, copy_stream: Optional[torch.cuda.Stream] = None,
+                           forced_sel: Optional[torch.Tensor] = None, final_hidden=None, sel_out=None,
+                           ws: Optional[torch.Tensor] = None, timings: bool = False):
+    """kvb_selective_prefill_host: chunk caches in pinned host memory, ingested layer by layer
+    on `copy_stream` under the compute on the current stream."""
+    dev = token_ids.device
+    if final_hidden is None:
+        final_hidden = torch.empty(max(n_query, 1), cfg.hidden, dtype=torch.float32, device=dev)
+    if sel_out is None:
+        sel_out = torch.empty(max(n_ctx, 1), dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = torch.zeros(workspace_size_pipelined(cfg, n_ctx + n_query, n_ctx), dtype=torch.uint8, device=dev)
+    if copy_stream is None:
+        copy_stream = torch.cuda.Stream(device=dev)
+    cache = kv_cache_struct(cache_k, cache_v)
+    t = Timings()
+    _call("kvb_selective_prefill_host", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct),
+          _host_ptr(k_chunks_host, torch.bfloat16, "k_chunks_host"), _host_ptr(v_chunks_host, torch.float16, "v_chunks_host"),
+          C.byref(cache), _ptr(token_ids, torch.int32, "token_ids"), _ptr(chunk_start, torch.int32, "chunk_start"),
+          chunk_start.numel() - 1, n_ctx, n_query, r, check_layer,
+          _ptr(forced_sel, torch.int32, "forced_sel"), forced_sel.numel() if forced_sel is not None else 0,
+          _ptr(final_hidden, torch.float32, "final_hidden"), _ptr(sel_out, torch.int32, "sel_out"),
+          C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream(), copy_stream.cuda_stream)
     return final_hidden[:n_query], sel_out, (t.as_dict() if timings else None)
 
 

@@ -240,3 +240,22 @@ def test_headline_full_ratio_equals_dense_prefill(kvb, headline):
     torch.cuda.synchronize()
     assert torch.equal(fh, fh2) and torch.equal(ck, ck2) and torch.equal(cv, cv2)
     assert torch.isfinite(fh).all()
+
+
+def test_headline_pipelined_ingest_equals_device_resident(kvb, headline):
+    h = headline
+    ck, cv = _cache()
+    fh, sel, _ = kvb.selective_prefill(h["cfg"], h["model"], h["rope"], h["kch"], h["vch"], ck, cv, h["toks"],
+                                       h["dstarts"], N_CTX, WL.n_query, WL.r, 1, ws=h["ws"])
+    hk = torch.empty(h["kch"].shape, dtype=h["kch"].dtype, pin_memory=True)
+    hv = torch.empty(h["vch"].shape, dtype=h["vch"].dtype, pin_memory=True)
+    hk.copy_(h["kch"])
+    hv.copy_(h["vch"])
+    ck2, cv2 = _cache()
+    wsp = torch.zeros(kvb.workspace_size_pipelined(h["cfg"], N, N_CTX), dtype=torch.uint8, device="cuda")
+    fh2, sel2, _ = kvb.selective_prefill_host(h["cfg"], h["model"], h["rope"], hk, hv, ck2, cv2, h["toks"],
+                                              h["dstarts"], N_CTX, WL.n_query, WL.r, 1, ws=wsp)
+    torch.cuda.synchronize()
+    assert kvb.device_status(wsp) == 0
+    k = blend.num_selected(WL.r, N_CTX)
+    assert torch.equal(fh, fh2) and torch.equal(sel[:k], sel2[:k]) and torch.equal(ck, ck2) and torch.equal(cv, cv2)

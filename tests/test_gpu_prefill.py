@@ -204,3 +204,25 @@ def test_repeatable_bitwise(kvb, case):
         outs.append((fh.clone(), sel[:k].clone(), ck.clone(), cv.clone()))
     for o in outs[1:]:
         assert all(torch.equal(a, b) for a, b in zip(o, outs[0]))
+
+
+def test_pipelined_host_ingest_equals_device_resident(kvb, case):
+    """Chunk caches in pinned host memory, ingested layer by layer on a copy stream
+    (Sec. 3.4), give bit-identical results to the device-resident call."""
+    ck, cv = case.new_cache()
+    fh, sel, _ = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks,
+                                       case.dstarts, case.n_ctx, case.nq, case.wl.r, 1, ws=case.ws)
+    hk = torch.empty(case.kch.shape, dtype=case.kch.dtype, pin_memory=True)
+    hv = torch.empty(case.vch.shape, dtype=case.vch.dtype, pin_memory=True)
+    hk.copy_(case.kch)
+    hv.copy_(case.vch)
+    ck2, cv2 = case.new_cache()
+    fh2, sel2, t = kvb.selective_prefill_host(case.cfg, case.model, case.rope, hk, hv, ck2, cv2, case.dtoks,
+                                              case.dstarts, case.n_ctx, case.nq, case.wl.r, 1, timings=True)
+    torch.cuda.synchronize()
+    k = blend.num_selected(case.wl.r, case.n_ctx)
+    assert torch.equal(fh, fh2) and torch.equal(sel[:k], sel2[:k])
+    assert torch.equal(ck, ck2) and torch.equal(cv, cv2)
+    with pytest.raises(ValueError):   # pageable memory is refused by the binding
+        kvb.selective_prefill_host(case.cfg, case.model, case.rope, hk.clone(), hv, ck2, cv2, case.dtoks,
+                                   case.dstarts, case.n_ctx, case.nq, case.wl.r, 1)
