@@ -62,6 +62,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=2, help="timed end-to-end steps (0: skip)")
     ap.add_argument("--cpu-rows", type=int, default=512, help="rows in the oracle's timed sample")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="64k-context sweep: r x chunk size, per-kernel times (prints one JSON line per point)")
     return ap.parse_args()
 
 
@@ -375,6 +377,51 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         print(json.dumps(out))
 
 
+def run_sweep(args) -> None:
+    """The 64k-context sweep: 32 layers, chunk sizes 256/512/1024/2048 (count adjusted to fill
+    65,536 context tokens) + 128 query tokens, r in {0.05, 0.10, 0.15, 0.25, 0.5, 1.0}; per point
+    the TTFT and the per-kernel times of re-align, HKVD (deviation + top-k), row GEMMs and
+    sparse-query attention."""
+    import torch
+    from paper_2609_09768_gb300 import build, synth, workload
+    from paper_2609_09768_gb300 import kvblend as kvb
+
+    build.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    shape = synth.LLAMA8B
+    cfg = kvb.config(shape)
+    nq, n_ctx = 128, 65536
+    N, L = n_ctx + nq, shape.n_layers
+    weights = workload.device_model(shape, seed=0, device=dev, draw_on_device=True)
+    model = kvb.Model(weights)
+    toks = synth.make_tokens(shape, N, 1).to(dev)
+    rope = kvb.RopeTable(cfg, N, dev)
+    ws = kvb.workspace(cfg, N, dev)
+    ck = torch.empty(L, N, shape.n_kv_heads, shape.head_dim, dtype=torch.bfloat16, device=dev)
+    cv = torch.empty(L, N, shape.n_kv_heads, shape.head_dim, dtype=torch.float16, device=dev)
+    fh = torch.empty(nq, shape.hidden, dtype=torch.float32, device=dev)
+    sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
+    for chunk in (256, 512, 1024, 2048):
+        starts = synth.chunk_starts_equal(n_ctx // chunk, chunk)
+        dstarts = torch.tensor(starts, dtype=torch.int32, device=dev)
+        kch, vch = workload.chunk_caches(cfg, model, rope, toks[:n_ctx], starts, ws=ws)
+        for r in (0.05, 0.10, 0.15, 0.25, 0.5, 1.0):
+            run = lambda: kvb.selective_prefill(cfg, model, rope, kch, vch, ck, cv, toks, dstarts, n_ctx, nq, r, 1,
+                                                final_hidden=fh, sel_out=sel, ws=ws, timings=True)[2]
+            for _ in range(max(1, args.warmup - 1)):
+                run()
+            reps = [run() for _ in range(max(1, min(args.steps, 3)))]
+            avg = {k: statistics.mean(t[k] for t in reps) for k in reps[0]}
+            print(json.dumps({"sweep": "l8b-32L-64k", "chunk": chunk, "n_chunks": n_ctx // chunk, "r": r,
+                              "k": int(avg["n_selected"]), "ttft_ms": round(avg["total_ms"], 2),
+                              "realign_ms": round(avg["realign_ms"], 3), "hkvd_ms": round(avg["hkvd_ms"], 3),
+                              "gemm_ms": round(avg["gemm_ms"], 2),
+                              "attn_sel_ms": round(avg["attn_sel_ms"], 2),
+                              "attn_dense_ms": round(avg["attn_dense_ms"], 2)}), flush=True)
+        del kch, vch
+    assert kvb.device_status(ws) == 0
+
+
 def main():
     args = parse()
     from paper_2609_09768_gb300 import synth
@@ -383,6 +430,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
         run_reference(args, wl, rank, world)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
     import torch
     if world > 1:

@@ -121,6 +121,7 @@ typedef struct kvb_timings {
     float attn_dense_ms;  /* attention launches of the dense layers                  */
     float attn_sel_ms;    /* attention launches of the selective layers              */
     float gemm_ms;        /* all GEMM launches                                        */
+    float hkvd_ms;        /* deviation + top-k launches                               */
     int32_t n_attn_dense, n_attn_sel, n_gemm;
     int32_t n_launches;   /* kernels this call launched                              */
     int64_t n_selected;   /* k = number of recomputed context rows                   */

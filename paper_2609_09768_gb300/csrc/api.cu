@@ -200,7 +200,7 @@ static void inv_freq(const kvb_config* c, double* w) {
 namespace {
 
 // Per-launch CUDA event pairs around the tensor-core kernels (only when timings are asked for).
-enum ProfKind { PK_ATTN_DENSE = 0, PK_ATTN_SEL = 1, PK_GEMM = 2, PK_COUNT = 3 };
+enum ProfKind { PK_ATTN_DENSE = 0, PK_ATTN_SEL = 1, PK_GEMM = 2, PK_HKVD = 3, PK_COUNT = 4 };
 struct Prof {
     cudaStream_t st = nullptr;
     std::vector<cudaEvent_t> ev;
@@ -338,6 +338,7 @@ static void fill_kernel_times(const Prof& prof, kvb_timings* t, int64_t launches
     t->attn_dense_ms = ms[PK_ATTN_DENSE];
     t->attn_sel_ms = ms[PK_ATTN_SEL];
     t->gemm_ms = ms[PK_GEMM];
+    t->hkvd_ms = ms[PK_HKVD];
     t->n_attn_dense = n[PK_ATTN_DENSE];
     t->n_attn_sel = n[PK_ATTN_SEL];
     t->n_gemm = n[PK_GEMM];
@@ -718,7 +719,9 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
                 p.status = w.status;
                 KVB_TRY(gemm(c, p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr));
                 KVB_TRY(wait_layer(lc));
+                const int hp = c.prof ? c.prof->begin(PK_HKVD) : -1;
                 KVB_TRY(launch_hkvd(w.k_fresh, kvd, kc(lc), kvd, n_ctx, (int)kvd, k, w.sel, w.dev, w.topk, c.st));
+                if (c.prof) c.prof->end(hp);
             }
             sel = w.sel;
         }

@@ -37,26 +37,44 @@ realign_kernel(const float* __restrict__ cos_t, const float* __restrict__ sin_t,
         const float cs[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
         const float sn[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
         const int64_t off = t * Hkv * D + h * D + gi * 8;
-        for (int l = 0; l < n_layers; ++l) {
-            const uint4 a = *reinterpret_cast<const uint4*>(k_src + l * src_ls + off);
-            const uint4 b = *reinterpret_cast<const uint4*>(k_src + l * src_ls + off + D / 2);
-            const uint32_t av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
-            uint32_t ra[4], rb[4];
+        // four layers' loads in flight before any store (memory-level parallelism)
+        constexpr int U = 4;
+        for (int l0 = 0; l0 < n_layers; l0 += U) {
+            uint4 ka[U], kb[U], va[U], vb[U];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float a0 = bf16_lo(av[e]), a1 = bf16_hi(av[e]);
-                const float b0 = bf16_lo(bv[e]), b1 = bf16_hi(bv[e]);
-                const float c_0 = cs[2 * e], c_1 = cs[2 * e + 1], s_0 = sn[2 * e], s_1 = sn[2 * e + 1];
-                ra[e] = pack_bf16(a0 * c_0 - b0 * s_0, a1 * c_1 - b1 * s_1);
-                rb[e] = pack_bf16(b0 * c_0 + a0 * s_0, b1 * c_1 + a1 * s_1);
+            for (int u = 0; u < U; ++u) {
+                if (l0 + u < n_layers) {
+                    const int64_t o = (int64_t)(l0 + u) * src_ls + off;
+                    ka[u] = __ldcs(reinterpret_cast<const uint4*>(k_src + o));
+                    kb[u] = __ldcs(reinterpret_cast<const uint4*>(k_src + o + D / 2));
+                    if (copy_v) {
+                        va[u] = __ldcs(reinterpret_cast<const uint4*>(v_src + o));
+                        vb[u] = __ldcs(reinterpret_cast<const uint4*>(v_src + o + D / 2));
+                    }
+                }
             }
-            *reinterpret_cast<uint4*>(k_dst + l * dst_ls + off) = make_uint4(ra[0], ra[1], ra[2], ra[3]);
-            *reinterpret_cast<uint4*>(k_dst + l * dst_ls + off + D / 2) = make_uint4(rb[0], rb[1], rb[2], rb[3]);
-            if (copy_v) {
-                *reinterpret_cast<uint4*>(v_dst + l * dst_ls + off) =
-                    *reinterpret_cast<const uint4*>(v_src + l * src_ls + off);
-                *reinterpret_cast<uint4*>(v_dst + l * dst_ls + off + D / 2) =
-                    *reinterpret_cast<const uint4*>(v_src + l * src_ls + off + D / 2);
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                if (l0 + u < n_layers) {
+                    const uint32_t av[4] = {ka[u].x, ka[u].y, ka[u].z, ka[u].w};
+                    const uint32_t bv[4] = {kb[u].x, kb[u].y, kb[u].z, kb[u].w};
+                    uint32_t ra[4], rb[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a0 = bf16_lo(av[e]), a1 = bf16_hi(av[e]);
+                        const float b0 = bf16_lo(bv[e]), b1 = bf16_hi(bv[e]);
+                        const float c_0 = cs[2 * e], c_1 = cs[2 * e + 1], s_0 = sn[2 * e], s_1 = sn[2 * e + 1];
+                        ra[e] = pack_bf16(a0 * c_0 - b0 * s_0, a1 * c_1 - b1 * s_1);
+                        rb[e] = pack_bf16(b0 * c_0 + a0 * s_0, b1 * c_1 + a1 * s_1);
+                    }
+                    const int64_t o = (int64_t)(l0 + u) * dst_ls + off;
+                    __stcs(reinterpret_cast<uint4*>(k_dst + o), make_uint4(ra[0], ra[1], ra[2], ra[3]));
+                    __stcs(reinterpret_cast<uint4*>(k_dst + o + D / 2), make_uint4(rb[0], rb[1], rb[2], rb[3]));
+                    if (copy_v) {
+                        __stcs(reinterpret_cast<uint4*>(v_dst + o), va[u]);
+                        __stcs(reinterpret_cast<uint4*>(v_dst + o + D / 2), vb[u]);
+                    }
+                }
             }
         }
     }

@@ -59,7 +59,7 @@ class KVCache(C.Structure):
 class Timings(C.Structure):
     _fields_ = [("total_ms", c_f32), ("realign_ms", c_f32), ("dense_ms", c_f32), ("select_ms", c_f32),
                 ("selective_ms", c_f32), ("final_ms", c_f32), ("attn_dense_ms", c_f32), ("attn_sel_ms", c_f32),
-                ("gemm_ms", c_f32), ("n_attn_dense", c_i32), ("n_attn_sel", c_i32), ("n_gemm", c_i32),
+                ("gemm_ms", c_f32), ("hkvd_ms", c_f32), ("n_attn_dense", c_i32), ("n_attn_sel", c_i32), ("n_gemm", c_i32),
                 ("n_launches", c_i32), ("n_selected", c_i64), ("n_rows", c_i64)]
 
     def as_dict(self) -> dict:
