@@ -174,12 +174,15 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     if (!mbar_wait(&k_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status)) break;
                     if (j >= 2 && !mbar_wait(&s_free[b], ((j - 2) >> 1) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
-                    const uint32_t kb = k0 + st * S::KV_BYTES;
+                    // descriptor built once per tile; constant steps inside the unrolled loop keep
+                    // the issuing thread ahead of the 64-cycle MMAs
+                    const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
+                    const uint32_t sd = tmem_base + COL_S + b * KT_ROWS, qa = tmem_base + COL_Q;
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
                         // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
-                        mma_f16_ts(tmem_base + COL_S + b * KT_ROWS, tmem_base + COL_Q + kk * 8,
-                                   sdesc_sw128(kb + (kk >> 2) * S::CHUNK + (kk & 3) * 32, 16, 1024), IDESC_S, kk > 0);
+                        mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32), IDESC_S,
+                                   kk > 0 ? 1u : 0u);
                     }
                     mma_commit(&k_empty[st]);
                     mma_commit(&s_full[b]);
@@ -189,12 +192,13 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     if (!mbar_wait(p_full, i & 1, abort_flag, p.status)) break;
                     if (!mbar_wait(&v_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
-                    const uint32_t vb = v0 + st * S::KV_BYTES;
+                    const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
+                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_P;
+                    mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
 #pragma unroll
-                    for (int kk = 0; kk < KT_ROWS / 16; ++kk) {
+                    for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
                         // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
-                        mma_f16_ts(tmem_base + COL_O, tmem_base + COL_P + kk * 8,
-                                   sdesc_sw128(vb + kk * 16 * 128, S::CHUNK, 1024), IDESC_O, (i > 0) || (kk > 0));
+                        mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
                     }
                     mma_commit(&v_empty[st]);
                     mma_commit(pv_done);

@@ -206,6 +206,10 @@ KVB_DEV uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
     return d;
 }
 
+// Advance a descriptor's start address by `bytes` (a multiple of 16 that keeps the
+// address inside shared memory, so the 14-bit field does not carry).
+__host__ __device__ constexpr uint64_t sdesc_add(uint64_t desc, uint32_t bytes) { return desc + (bytes >> 4); }
+
 // 32 lanes x 32-bit, 16 consecutive columns: thread t gets lane (base lane + t).
 KVB_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile(

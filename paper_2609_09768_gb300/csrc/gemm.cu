@@ -144,12 +144,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                     if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(smem + stage * STAGE_BYTES);
-                    const uint32_t b0 = a0 + A_BYTES;
+                    // descriptors built once per stage; each K step of 16 advances 32 bytes
+                    const uint64_t ad = sdesc_sw128(a0, 16, 1024), bd = sdesc_sw128(a0 + A_BYTES, 16, 1024);
+                    mma_bf16_ss(d, ad, bd, IDESC, kb != 0);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {
-                        mma_bf16_ss(d, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), IDESC,
-                                    (kb | k) != 0);
-                    }
+                    for (int k = 1; k < BK / 16; ++k)
+                        mma_bf16_ss(d, sdesc_add(ad, k * 32), sdesc_add(bd, k * 32), IDESC, 1u);
                     mma_commit(&empty[stage]);
                     if (++stage == STAGES) { stage = 0; phase ^= 1; }
                 }
