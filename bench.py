@@ -222,11 +222,25 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     cv = torch.empty(L, N, Hkv, D, dtype=torch.float16, device=dev)
     fh = torch.empty(nq, H, dtype=torch.float32, device=dev)
     sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
+    lm = synth.make_lm_head(shape, 0, dev)
+    tok = torch.empty(1, dtype=torch.int32, device=dev)
+    lm_ws = torch.zeros(512, dtype=torch.uint8, device=dev)
+    lm_ev = []
     torch.cuda.synchronize()
 
+    def first_token():
+        """Logits of the last query row over the vocabulary and their argmax."""
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        kvb.lm_head_argmax(cfg, lm, fh[nq - 1:], tokens=tok, ws=lm_ws)
+        b.record()
+        lm_ev.append((a, b))
+
     def step(rr=r, timings=True):
-        return kvb.selective_prefill(cfg, model, rope, kch, vch, ck, cv, toks, dstarts, n_ctx, nq, rr, 1,
-                                     final_hidden=fh, sel_out=sel, ws=ws, timings=timings)[2]
+        t = kvb.selective_prefill(cfg, model, rope, kch, vch, ck, cv, toks, dstarts, n_ctx, nq, rr, 1,
+                                  final_hidden=fh, sel_out=sel, ws=ws, timings=timings)[2]
+        first_token()
+        return t
 
     def barrier():
         if world > 1:
@@ -240,6 +254,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     barrier()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    lm_ev.clear()
     e0.record()
     tims = [step() for _ in range(args.steps)]
     e1.record()
@@ -272,6 +287,11 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         "attn_dense": {"ms": avg("attn_dense_ms"), "launches": int(tims[-1]["n_attn_dense"]), "flop": attn_dense_flop},
         "gemm": {"ms": avg("gemm_ms"), "launches": int(tims[-1]["n_gemm"]), "flop": gemm_flop},
     }
+    lm_ms = statistics.mean(a.elapsed_time(b) for a, b in lm_ev[:args.steps])
+    lm_bytes = float(shape.vocab * H * 2)
+    lm_head = {"ms": round(lm_ms, 4), "launches": 2, "bytes": lm_bytes,
+               "gbs": round(lm_bytes / (lm_ms * 1e-3) / 1e9, 1),
+               "frac_of_hbm": round(lm_bytes / (lm_ms * 1e-3) / 1e9 / pk["hbm_gbs"], 4)}
     for v in kern.values():
         v["tflops"] = v["flop"] / (v["ms"] * 1e-3) / 1e12 if v["ms"] > 0 else None
         v["frac_of_sustained_peak"] = (v["tflops"] / pk["bf16_sustained"]) if v["tflops"] else None
@@ -311,6 +331,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         hv = torch.empty(vch.shape, dtype=vch.dtype, pin_memory=True)
         ht = torch.empty(toks.shape, dtype=toks.dtype, pin_memory=True)
         hf = torch.empty(fh.shape, dtype=fh.dtype, pin_memory=True)
+        htok = torch.empty(tok.shape, dtype=tok.dtype, pin_memory=True)
         hk.copy_(kch); hv.copy_(vch); ht.copy_(toks)
         td = torch.empty_like(toks)
         wsp = torch.zeros(kvb.workspace_size_pipelined(cfg, N, n_ctx), dtype=torch.uint8, device=dev)
@@ -321,7 +342,9 @@ def run_ours(args, wl, rank: int, world: int) -> None:
             td.copy_(ht, non_blocking=True)
             kvb.selective_prefill_host(cfg, model, rope, hk, hv, ck, cv, td, dstarts, n_ctx, nq, r, 1,
                                        copy_stream=cs, final_hidden=fh, sel_out=sel, ws=wsp)
+            kvb.lm_head_argmax(cfg, lm, fh[nq - 1:], tokens=tok, ws=lm_ws)
             hf.copy_(fh, non_blocking=True)
+            htok.copy_(tok, non_blocking=True)
 
         e2e_step()
         torch.cuda.synchronize()
@@ -339,7 +362,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         h2d_ms = a.elapsed_time(b)
         h2d = hk.numel() * 2 + hv.numel() * 2 + ht.numel() * 4
         e2e = {"value": round(e2e_ms, 3), "unit": "ms", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(hf.numel() * 4), "path": "kvb_selective_prefill_host (layer-wise ingest)",
+               "d2h_bytes_per_step": int(hf.numel() * 4 + htok.numel() * 4), "path": "kvb_selective_prefill_host (layer-wise ingest)",
                "bare_h2d_ms": round(h2d_ms, 2), "bare_h2d_gbs": round(h2d / (h2d_ms * 1e-3) / 1e9, 1)}
         del hk, hv, kd, wsp
 
@@ -369,9 +392,10 @@ def run_ours(args, wl, rank: int, world: int) -> None:
             "r1_dense": r1,
             "ttft_reduction_vs_r1": (round(1.0 - ms / r1["ttft_ms"], 4) if r1 else None),
             "algorithmic_tflops": round(total_flop / (ms * 1e-3) / 1e12, 2),
-            "stages_ms": stages, "kernels": kdict,
+            "stages_ms": stages, "kernels": dict(kdict, first_token_lm_head=lm_head),
+            "first_token": int(tok.item()),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": int(sum(t["n_launches"] for t in tims)),
+            "gpu_launches": int(sum(t["n_launches"] for t in tims)) + 2 * args.steps,
             "clocks": clk,
         }
         print(json.dumps(out))

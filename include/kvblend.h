@@ -338,6 +338,18 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
                             float* final_hidden, int64_t n_out,
                             kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
 
+/* First token (the "first token" that closes time-to-first-token, Sec. 4.3): for n rows
+ * of final hidden states h (fp32 [n][H], already through the final RMSNorm),
+ *   logits[r][v] = h[r] . W[v]      (W: lm_head, bf16 [vocab][H]; fp32 accumulation)
+ *   tokens[r]    = argmax_v logits[r][v], ties to the lower token id.
+ * logits_out: fp32 [n][vocab] or NULL; tokens_out: int32 [n].  1 <= n <=
+ * KVB_LMHEAD_MAX_ROWS, H <= 8192, H % 8 == 0.  Workspace: >= 256 + 8 * n bytes (the
+ * status word, then one 64-bit argmax slot per row that the call clears).  Errors:
+ * INVALID_ARG, WORKSPACE. */
+#define KVB_LMHEAD_MAX_ROWS 4
+kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, const float* hidden, int32_t n,
+                              float* logits_out, int32_t* tokens_out, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, then read and clear the device status word that kernels using
  * workspace `ws` write when a bounded wait runs out.  *code_out receives KVB_OK or
  * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */

@@ -186,3 +186,10 @@ def selective_prefill(s: Shape, layers: Sequence[dict], x0, chunk_starts: Sequen
     fh = q_rows if final_norm is None else rmsnorm(q_rows, final_norm, s.rms_eps)
     return {"final_hidden": fh, "sel": sel, "dev": dev, "rows": rows,
             "layer_out": layer_out, "k": kc, "v": vc}
+
+
+def first_token(hidden, lm_head) -> tuple:
+    """The first generated token (greedy decoding, Sec. 4): logits = h W^T over the vocabulary,
+    token = argmax (the lowest id among equal maxima).  hidden: [n, H] final hidden states."""
+    logits = as64(hidden) @ as64(lm_head).T
+    return np.argmax(logits, axis=-1).astype(np.int64), logits

@@ -800,6 +800,23 @@ kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, i
     return KVB_OK;
 }
 
+kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, const float* hidden, int32_t n,
+                              float* logits_out, int32_t* tokens_out, void* ws, size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    KVB_TRY(check_cfg(cfg));
+    if (n < 1 || n > KVB_LMHEAD_MAX_ROWS || cfg->vocab < 1 || cfg->hidden > 8192 || cfg->hidden % 8)
+        return fail(KVB_ERR_INVALID_ARG, "lm head: need 1 <= n <= %d rows, vocab >= 1, hidden <= 8192",
+                    KVB_LMHEAD_MAX_ROWS);
+    KVB_TRY(check_ptr(lm_head, "lm_head"));
+    KVB_TRY(check_ptr(hidden, "hidden"));
+    KVB_TRY(check_ptr(tokens_out, "tokens_out"));
+    if (logits_out) KVB_TRY(check_ptr(logits_out, "logits_out"));
+    if (!ws || ws_bytes < 256 + 8 * (size_t)n) return fail(KVB_ERR_WORKSPACE, "lm head: workspace too small");
+    auto* keys = reinterpret_cast<unsigned long long*>(static_cast<char*>(ws) + 256);
+    return launch_lmhead(lm_head, cfg->vocab, cfg->hidden, hidden, n, logits_out, keys, tokens_out,
+                         static_cast<cudaStream_t>(stream));
+}
+
 kvb_status kvb_debug_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
     g_err[0] = 0;
     if (!ws || ws_bytes < 256 || limit_ns < 1000 || limit_ns > 4000000000ll)

@@ -96,6 +96,8 @@ kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t
                        cudaStream_t st);
 
 kvb_status launch_wait_timeout(int* status, uint64_t limit_ns, cudaStream_t st);
+kvb_status launch_lmhead(const uint16_t* W, int64_t vocab, int H, const float* x, int n, float* logits,
+                         unsigned long long* keys, int32_t* tokens, cudaStream_t st);
 
 // ---------------------------------------------------------------- workspace
 // Layout of a caller workspace for up to n rows.

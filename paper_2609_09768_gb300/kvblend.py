@@ -96,6 +96,7 @@ _SIGS = {
                                  c_vp, c_i64, P(Timings), c_vp, c_sz, c_vp]),
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
     "kvb_debug_wait_timeout": (c_i32, [c_vp, c_sz, c_i64, c_vp]),
+    "kvb_lm_head_argmax": (c_i32, [P(Config), c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_sz, c_vp]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -206,6 +207,24 @@ def workspace_size(cfg: Config, n_rows: int) -> int:
 def workspace(cfg: Config, n_rows: int, device="cuda") -> torch.Tensor:
     """A zeroed workspace (the zeroed head is the device status word)."""
     return torch.zeros(workspace_size(cfg, n_rows), dtype=torch.uint8, device=device)
+
+
+LMHEAD_MAX_ROWS = 4
+
+
+def lm_head_argmax(cfg: Config, lm_head: torch.Tensor, hidden: torch.Tensor, logits: Optional[torch.Tensor] = None,
+                   tokens: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None):
+    """First-token logits and argmax for up to LMHEAD_MAX_ROWS rows of final hidden states."""
+    n = hidden.shape[0]
+    dev = hidden.device
+    if tokens is None:
+        tokens = torch.empty(n, dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = torch.zeros(256 + 8 * LMHEAD_MAX_ROWS, dtype=torch.uint8, device=dev)
+    _call("kvb_lm_head_argmax", C.byref(cfg), _ptr(lm_head, torch.bfloat16, "lm_head"),
+          _ptr(hidden, torch.float32, "hidden"), n, _ptr(logits, torch.float32, "logits"),
+          _ptr(tokens, torch.int32, "tokens"), _ptr(ws), ws.numel(), _stream())
+    return tokens, logits
 
 
 def debug_wait_timeout(ws: torch.Tensor, limit_ns: int) -> None:

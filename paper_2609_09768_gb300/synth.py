@@ -27,7 +27,7 @@ import torch
 
 __all__ = [
     "ModelShape", "Workload", "SHAPES", "WORKLOADS", "tensor_seed",
-    "make_layer_weights", "make_embed", "make_model", "make_tokens",
+    "make_layer_weights", "make_embed", "make_lm_head", "make_model", "make_tokens",
     "chunk_starts_equal", "randn_bf16",
 ]
 
@@ -152,6 +152,11 @@ def make_layer_weights(shape: ModelShape, layer: int, seed: int = 0,
 
 def make_embed(shape: ModelShape, seed: int = 0, device: str | torch.device = "cpu") -> torch.Tensor:
     return randn_bf16((shape.vocab, shape.hidden), tensor_seed(seed, -1, "embed"), 1.0, device)
+
+
+def make_lm_head(shape: ModelShape, seed: int = 0, device: str | torch.device = "cpu") -> torch.Tensor:
+    """Output projection [vocab][hidden], N(0, 0.02) rounded to bf16."""
+    return randn_bf16((shape.vocab, shape.hidden), tensor_seed(seed, -3, "lm_head"), 0.02, device)
 
 
 def make_model(shape: ModelShape, seed: int = 0, device: str | torch.device = "cpu") -> dict:

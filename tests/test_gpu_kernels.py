@@ -233,3 +233,87 @@ def test_bounded_wait_reports_timeout_and_context_survives(kvb):
     kvb.kv_scatter(dev(kr), dev(kr.to(torch.float16)), dev(idx), kd, vd)
     torch.cuda.synchronize()
     assert torch.equal(kd.cpu()[idx.long()], kr)
+
+
+# ------------------------------------------------------------------------------------- first token
+
+def _lm_head_bound(h64, w64):
+    """Worst-case error of an fp32 dot product of length H against the exact value:
+    gamma_H * sum_i |w_i x_i| with gamma_H = H u / (1 - H u), u = 2^-24 (round to nearest)."""
+    u = 2.0 ** -24
+    H = h64.shape[1]
+    gamma = H * u / (1 - H * u)
+    return gamma * (np.abs(h64) @ np.abs(w64).T)          # [n, vocab]
+
+
+def _check_first_token(kvb, shape, h, w, with_logits=True):
+    n = h.shape[0]
+    cfg = kvb.config(shape)
+    logits = torch.empty(n, shape.vocab, dtype=torch.float32, device="cuda") if with_logits else None
+    tok, _ = kvb.lm_head_argmax(cfg, dev(w), dev(h), logits)
+    torch.cuda.synchronize()
+    tok = tok.cpu().numpy().astype(np.int64)
+    h64, w64 = np64(h), np64(w)
+    want_tok, want_logits = blend.first_token(h64, w64)
+    bound = _lm_head_bound(h64, w64)
+    if with_logits:
+        got = np64(logits.cpu())
+        assert np.all(np.abs(got - want_logits) <= bound), np.abs(got - want_logits).max()
+    rows = np.arange(n)
+    # the chosen token's exact logit is within two error bounds of the exact maximum ...
+    assert np.all(want_logits[rows, tok] >= want_logits[rows, want_tok] - bound[rows, tok] - bound[rows, want_tok])
+    # ... and is the oracle's token wherever the top-two gap exceeds those bounds
+    srt = np.sort(want_logits, axis=1)
+    gap = srt[:, -1] - srt[:, -2] if shape.vocab > 1 else np.full(n, np.inf)
+    clear = gap > 2 * bound.max(axis=1)
+    assert np.array_equal(tok[clear], want_tok[clear])
+    return tok, want_tok
+
+
+@pytest.mark.parametrize("vocab,hidden,n", [
+    (128256, 4096, 1),          # Llama-3.1-8B output layer, one query row
+    (128256, 4096, 4),          # the most rows one call takes
+    (50001, 4096, 3),           # ragged vocabulary
+    (1024, 256, 2),
+    (1, 256, 1),                # a one-token vocabulary
+])
+def test_lm_head_argmax_matches_oracle(kvb, vocab, hidden, n):
+    shape = synth.ModelShape(hidden, 4, 2, 64, 4 * hidden, 1, vocab)
+    w = synth.randn_bf16((vocab, hidden), 501 + n, 0.02)
+    h = torch.randn(n, hidden, generator=torch.Generator().manual_seed(vocab + n), dtype=torch.float64).float()
+    _check_first_token(kvb, shape, h, w)
+    if vocab > 1:
+        _check_first_token(kvb, shape, h, w, with_logits=False)
+
+
+def test_lm_head_argmax_ties_and_negative_logits(kvb):
+    """Equal weight rows give bit-equal fp32 logits (same reduction order for every row);
+    the lowest id must win.  All-negative logits exercise the sign handling of the key."""
+    vocab, hidden = 4099, 512
+    shape = synth.ModelShape(hidden, 4, 2, 64, 4 * hidden, 1, vocab)
+    w = synth.randn_bf16((vocab, hidden), 511, 0.02)
+    h = torch.randn(2, hidden, generator=torch.Generator().manual_seed(5), dtype=torch.float64).float()
+    # row 0: make token 3000 the clear winner, duplicated at ids 17 and 4098
+    w[3000] = (h[0].sign() * 0.05).to(torch.bfloat16)
+    w[17] = w[3000]
+    w[4098] = w[3000]
+    tok, _ = _check_first_token(kvb, shape, h, w)
+    assert tok[0] == 17
+    # all logits negative: W rows anti-aligned with h, the least negative wins
+    wn = -(h[1].sign() * (0.01 + 0.01 * torch.rand(vocab, 1, generator=torch.Generator().manual_seed(6)))).to(
+        torch.bfloat16)
+    tok, want = _check_first_token(kvb, shape, h[1:].contiguous(), wn.contiguous())
+    assert tok[0] == want[0]
+
+
+def test_lm_head_argmax_rejects_bad_arguments(kvb):
+    shape = synth.ModelShape(256, 4, 2, 64, 1024, 1, 64)
+    cfg = kvb.config(shape)
+    w = dev(synth.randn_bf16((64, 256), 3))
+    for n in (0, kvb.LMHEAD_MAX_ROWS + 1):
+        h = torch.zeros(n, 256, device="cuda")
+        with pytest.raises(kvb.KvbError):
+            kvb.lm_head_argmax(cfg, w, h, tokens=torch.empty(max(n, 1), dtype=torch.int32, device="cuda"))
+    with pytest.raises(kvb.KvbError):
+        kvb.lm_head_argmax(cfg, w, torch.zeros(1, 256, device="cuda"),
+                           ws=torch.zeros(64, dtype=torch.uint8, device="cuda"))

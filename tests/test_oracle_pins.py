@@ -442,3 +442,16 @@ def test_accum32_is_a_float32_accumulation_of_the_same_model():
     a = blend.full_prefill(Shape.of(shape, act_bf16=True), m["layers_np"], x0)["x"]
     b = blend.full_prefill(Shape.of(shape, act_bf16=True, accum32=True), m["layers_np"], x0)["x"]
     assert 0 < rel(a, b) < 1e-2
+
+
+def test_first_token_is_argmax_with_lowest_id_on_ties():
+    W = np.array([[1.0, 0.0], [0.0, 1.0], [1.0, 0.0], [0.5, 0.5]])
+    tok, logits = blend.first_token(np.array([[2.0, 1.0], [1.0, 1.0]]), W)
+    assert list(tok) == [0, 0]                      # row 0: ids 0 and 2 tie at 2 -> 0; row 1: all tie at 1 -> 0
+    assert np.allclose(logits, [[2, 1, 2, 1.5], [1, 1, 1, 1]])
+    rng = np.random.default_rng(13)
+    h, w = rng.standard_normal((3, 16)), rng.standard_normal((50, 16))
+    tok, logits = blend.first_token(h, w)
+    for r in range(3):
+        best = max(range(50), key=lambda v: (sum(h[r, d] * w[v, d] for d in range(16)), -v))
+        assert tok[r] == best
