@@ -64,6 +64,9 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--sweep", action="store_true",
                     help="64k-context sweep: r x chunk size, per-kernel times (prints one JSON line per point)")
+    ap.add_argument("--selectors", action="store_true",
+                    help="separator workload: TTFT and per-layer key-deviation histograms against the full "
+                         "prefill for plain concatenation, HKVD, EPIC and KVLink selections (one JSON line each)")
     return ap.parse_args()
 
 
@@ -446,6 +449,82 @@ def run_sweep(args) -> None:
     assert kvb.device_status(ws) == 0
 
 
+def run_selectors(args) -> None:
+    """Selections compared on a request with two zero-KV separator tokens between documents:
+    plain concatenation (r = 0), CacheBlend's HKVD at r, EPIC (20 rows from every separator)
+    and KVLink's rows (the separators).  Per selection: TTFT and, for every layer, the
+    histogram of per-token squared key differences of the blended cache against the
+    full prefill's cache (the quantity of the paper's deviation figures)."""
+    import numpy as np
+    import torch
+    from paper_2609_09768_gb300 import build, synth, workload
+    from paper_2609_09768_gb300 import kvblend as kvb
+
+    build.build()
+    wl = synth.WORKLOADS[args.workload if args.workload.endswith("_sep") else "l8b_124k_sep"]
+    dev = torch.device("cuda", torch.cuda.current_device())
+    shape = wl.shape
+    cfg = kvb.config(shape)
+    N, n_ctx, nq, L = wl.n_total, wl.n_ctx, wl.n_query, shape.n_layers
+    r = wl.r if args.r is None else args.r
+    model = kvb.Model(workload.device_model(shape, seed=0, device=dev, draw_on_device=True))
+    toks = wl.tokens(1, dev)
+    rope = kvb.RopeTable(cfg, N, dev)
+    ws = kvb.workspace(cfg, N, dev)
+    starts = wl.chunk_starts()
+    dstarts = torch.tensor(starts, dtype=torch.int32, device=dev)
+    kch, vch = workload.chunk_caches(cfg, model, rope, toks[:n_ctx], starts, ws=ws, zero_rows=wl.sep_rows())
+    shp = (L, N, shape.n_kv_heads, shape.head_dim)
+    ckf = torch.empty(shp, dtype=torch.bfloat16, device=dev)
+    cvf = torch.empty(shp, dtype=torch.float16, device=dev)
+    ck = torch.empty(shp, dtype=torch.bfloat16, device=dev)
+    cv = torch.empty(shp, dtype=torch.float16, device=dev)
+    fh = torch.empty(nq, shape.hidden, dtype=torch.float32, device=dev)
+    sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
+    seps = torch.tensor(wl.sep_starts(), dtype=torch.int32, device=dev)
+    epic, k_epic = kvb.window_select(seps, 20, n_ctx)
+    kvlink, k_kvlink = kvb.window_select(seps, wl.n_sep, n_ctx)
+    edges_l = [0.0] + [float(10.0 ** e) for e in np.arange(-4, 3.01, 0.5)]
+    edges = torch.tensor(edges_l, dtype=torch.float32, device=dev)
+    kd = shape.kv_dim
+
+    def run(rr, forced=None, cache=(ck, cv)):
+        return kvb.selective_prefill(cfg, model, rope, kch, vch, cache[0], cache[1], toks, dstarts, n_ctx, nq, rr, 1,
+                                     forced_sel=forced, final_hidden=fh, sel_out=sel, ws=ws, timings=True)[2]
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            t = fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps, t
+
+    full_ms, _ = timed(lambda: run(1.0, cache=(ckf, cvf)), 1)
+    print(json.dumps({"selectors": wl.name, "selection": "full prefill (r = 1)", "k": n_ctx,
+                      "ttft_ms": round(full_ms, 2)}), flush=True)
+    for name, rr, forced in (("concatenation (r = 0)", 0.0, None), (f"CacheBlend HKVD r = {r}", r, None),
+                             ("EPIC: 20 rows from every separator", 0.0, epic),
+                             ("KVLink rows: the separators", 0.0, kvlink)):
+        ms, t = timed(lambda: run(rr, forced), max(1, min(args.steps, 3)))
+        hist = {}
+        mean_dev = []
+        d = torch.empty(n_ctx, dtype=torch.float32, device=dev)
+        for l in range(1, L):
+            h = kvb.key_deviation_histogram(ck[l, :n_ctx].view(n_ctx, kd), ckf[l, :n_ctx].view(n_ctx, kd), edges,
+                                            dev_out=d)
+            mean_dev.append(round(float(d.mean()), 5))
+            if l in (1, 2, L // 2, L - 1):
+                hist[l] = h.cpu().tolist()
+        print(json.dumps({"selectors": wl.name, "selection": name, "k": int(t["n_selected"]),
+                          "ttft_ms": round(ms, 2), "ttft_vs_full": round(ms / full_ms, 4),
+                          "hist_edges": edges_l, "hist_by_layer": hist, "mean_dev_by_layer": mean_dev}), flush=True)
+    assert kvb.device_status(ws) == 0
+
+
 def main():
     args = parse()
     from paper_2609_09768_gb300 import synth
@@ -457,6 +536,9 @@ def main():
         return
     if args.sweep:
         run_sweep(args)
+        return
+    if args.selectors:
+        run_selectors(args)
         return
     import torch
     if world > 1:

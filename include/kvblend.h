@@ -350,6 +350,37 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
 kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, const float* hidden, int32_t n,
                               float* logits_out, int32_t* tokens_out, void* ws, size_t ws_bytes, void* stream);
 
+/* Fixed-position selection of the methods the paper compares against (Sec. 2 and
+ * Sec. 3.1): EPIC recomputes the 20 tokens that start at each separator position,
+ * KVLink the separator tokens themselves.  Writes the union of the windows
+ * [win_start[w], win_start[w] + window), cut to [0, n_ctx), as ascending context
+ * indices, and their count.  The result is meant for kvb_selective_prefill's forced_sel.
+ *   win_start: device int32 [n_win], any order, values may lie outside [0, n_ctx)
+ *   sel_out:   device int32, room for min(n_ctx, n_win * window) indices
+ *   k_out:     device int64 [1], the number of indices written
+ * 0 <= n_win, 0 <= window, n_win * window < 2^31, 0 <= n_ctx < 2^31.  Workspace:
+ * kvb_window_select_workspace_size bytes (the status word, then one flag byte per
+ * context row).  Errors: INVALID_ARG, WORKSPACE. */
+size_t kvb_window_select_workspace_size(int64_t n_ctx);
+kvb_status kvb_window_select(const int32_t* win_start, int32_t n_win, int32_t window, int64_t n_ctx, int32_t* sel_out,
+                             int64_t* k_out, void* ws, size_t ws_bytes, void* stream);
+
+/* Distribution of per-token squared key differences, as in the paper's figures of the
+ * deviation in the key entries (Sec. 3.2, Sec. 3.3):
+ *   dev[i] = sum over the kv_dim entries of (K_a[i] - K_b[i])^2   (bf16 in, fp32 sum)
+ *   hist[j] = #{ i : j == #{ e : dev[i] >= edges[e] } },  j = 0 .. n_edges
+ * so for ascending edges hist[0] counts dev < edges[0], hist[j] counts
+ * edges[j-1] <= dev < edges[j] and hist[n_edges] counts dev >= edges[n_edges-1].
+ *   k_a, k_b: device bf16, row i at k_a + i * ld_a (ld, kv_dim multiples of 8)
+ *   edges:    device fp32 [n_edges], 1 <= n_edges <= 1024
+ *   dev_out:  device fp32 [n] or NULL (then the workspace holds it)
+ *   hist_out: device int64 [n_edges + 1], cleared by the call
+ * Workspace: >= 256 bytes, plus 4 * n rounded up to 16 when dev_out is NULL.
+ * Errors: INVALID_ARG, WORKSPACE. */
+kvb_status kvb_key_deviation_histogram(const uint16_t* k_a, int64_t ld_a, const uint16_t* k_b, int64_t ld_b, int64_t n,
+                                       int32_t kv_dim, const float* edges, int32_t n_edges, float* dev_out,
+                                       int64_t* hist_out, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, then read and clear the device status word that kernels using
  * workspace `ws` write when a bounded wait runs out.  *code_out receives KVB_OK or
  * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */

@@ -111,7 +111,7 @@ def hkvd_deviation(k_fresh, k_cached) -> np.ndarray:
     """dev[i] = sum over kv heads h and dims d of (K_fresh[i,h,d] - K_cached[i,h,d])^2."""
     a = as64(k_fresh)
     b = as64(k_cached)
-    d = (a - b).reshape(a.shape[0], -1)
+    d = (a - b).reshape(a.shape[0], int(np.prod(a.shape[1:])))
     return np.sum(d * d, axis=1)
 
 
@@ -193,3 +193,42 @@ def first_token(hidden, lm_head) -> tuple:
     token = argmax (the lowest id among equal maxima).  hidden: [n, H] final hidden states."""
     logits = as64(hidden) @ as64(lm_head).T
     return np.argmax(logits, axis=-1).astype(np.int64), logits
+
+
+def zero_kv_rows(caches: dict, rows) -> dict:
+    """Separator tokens (Sec. 3.1, Sec. 4): two special tokens sit between consecutive
+    documents and their entries in the concatenated cache are all zero, K and V, every
+    layer.  Returns a copy of the caches {"k", "v"} ([L, N_ctx, Hkv, D]) with `rows` zeroed."""
+    k = as64(caches["k"]).copy()
+    v = as64(caches["v"]).copy()
+    rows = np.asarray(rows, dtype=np.int64)
+    k[:, rows] = 0.0
+    v[:, rows] = 0.0
+    return {"k": k, "v": v}
+
+
+def window_select(win_starts, window: int, n_ctx: int) -> np.ndarray:
+    """Fixed-position selection of the compared methods (Sec. 2, Sec. 3.1): EPIC recomputes
+    the `window` = 20 tokens that start at each separator position; KVLink recomputes
+    the separator tokens themselves (window = number of separator tokens).  The set is
+    the union of [s, s + window) over the window starts s, cut to [0, n_ctx), ascending."""
+    mark = [False] * n_ctx
+    for s in win_starts:
+        for i in range(int(s), int(s) + int(window)):
+            if 0 <= i < n_ctx:
+                mark[i] = True
+    return np.array([i for i in range(n_ctx) if mark[i]], dtype=np.int64)
+
+
+def deviation_histogram(dev, edges) -> np.ndarray:
+    """Distribution of per-token squared key differences (the figures of Sec. 3.2 and 3.3).
+    Each value d falls in bin j = #(edges e with d >= e); for ascending edges that is
+    counts[0] = #(d < edges[0]), counts[j] = #(edges[j-1] <= d < edges[j]),
+    counts[len(edges)] = #(d >= edges[-1]).  The comparisons are made in the precision
+    of `dev` and `edges` as given."""
+    dev = np.asarray(dev)
+    edges = np.asarray(edges)
+    counts = np.zeros(len(edges) + 1, dtype=np.int64)
+    for d in dev:
+        counts[sum(1 for e in edges if d >= e)] += 1
+    return counts

@@ -800,6 +800,55 @@ kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, i
     return KVB_OK;
 }
 
+static kvb_status check_ptr4(const void* p, const char* name) {
+    if (!p) return fail(KVB_ERR_INVALID_ARG, "%s is NULL", name);
+    if (reinterpret_cast<uintptr_t>(p) % 4) return fail(KVB_ERR_INVALID_ARG, "%s is not 4-byte aligned", name);
+    return KVB_OK;
+}
+
+static size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+size_t kvb_window_select_workspace_size(int64_t n_ctx) { return 256 + round16(n_ctx > 0 ? (size_t)n_ctx : 0); }
+
+kvb_status kvb_window_select(const int32_t* win_start, int32_t n_win, int32_t window, int64_t n_ctx, int32_t* sel_out,
+                             int64_t* k_out, void* ws, size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    if (n_win < 0 || window < 0 || n_ctx < 0 || n_ctx > 0x7FFFFFFF || (int64_t)n_win * window > 0x7FFFFFFF)
+        return fail(KVB_ERR_INVALID_ARG, "window select: need 0 <= n_win, window; n_win * window and n_ctx < 2^31");
+    if (n_win > 0) KVB_TRY(check_ptr4(win_start, "win_start"));
+    KVB_TRY(check_ptr4(sel_out, "sel_out"));
+    if (!k_out || reinterpret_cast<uintptr_t>(k_out) % 8) return fail(KVB_ERR_INVALID_ARG, "k_out NULL or misaligned");
+    const size_t need = kvb_window_select_workspace_size(n_ctx);
+    if (!ws || ws_bytes < need) return fail(KVB_ERR_WORKSPACE, "window select: workspace %zu < %zu", ws_bytes, need);
+    uint8_t* flags = static_cast<uint8_t*>(ws) + 256;
+    return launch_window_select(win_start, n_win, window, n_ctx, flags, sel_out, k_out,
+                                static_cast<cudaStream_t>(stream));
+}
+
+kvb_status kvb_key_deviation_histogram(const uint16_t* k_a, int64_t ld_a, const uint16_t* k_b, int64_t ld_b, int64_t n,
+                                       int32_t kv_dim, const float* edges, int32_t n_edges, float* dev_out,
+                                       int64_t* hist_out, void* ws, size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    if (n < 0 || n > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "deviation histogram: n out of range");
+    if (kv_dim <= 0 || kv_dim % 8 || ld_a < kv_dim || ld_b < kv_dim || ld_a % 8 || ld_b % 8)
+        return fail(KVB_ERR_INVALID_ARG, "deviation histogram: kv_dim and leading dims must be multiples of 8");
+    if (n_edges < 1 || n_edges > 1024) return fail(KVB_ERR_INVALID_ARG, "deviation histogram: 1 <= n_edges <= 1024");
+    KVB_TRY(check_ptr4(edges, "edges"));
+    if (!hist_out || reinterpret_cast<uintptr_t>(hist_out) % 8)
+        return fail(KVB_ERR_INVALID_ARG, "hist_out NULL or misaligned");
+    if (n > 0) {
+        KVB_TRY(check_ptr(k_a, "k_a"));
+        KVB_TRY(check_ptr(k_b, "k_b"));
+    }
+    if (dev_out) KVB_TRY(check_ptr4(dev_out, "dev_out"));
+    const size_t need = 256 + (dev_out ? 0 : round16((size_t)n * 4));
+    if (!ws || ws_bytes < need) return fail(KVB_ERR_WORKSPACE, "deviation histogram: workspace %zu < %zu", ws_bytes, need);
+    float* dev = dev_out ? dev_out : reinterpret_cast<float*>(static_cast<char*>(ws) + 256);
+    return launch_deviation_histogram(k_a, ld_a, k_b, ld_b, n, kv_dim, edges, n_edges, dev,
+                                      reinterpret_cast<unsigned long long*>(hist_out),
+                                      static_cast<cudaStream_t>(stream));
+}
+
 kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, const float* hidden, int32_t n,
                               float* logits_out, int32_t* tokens_out, void* ws, size_t ws_bytes, void* stream) {
     g_err[0] = 0;

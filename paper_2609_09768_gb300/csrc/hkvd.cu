@@ -158,6 +158,16 @@ kvb_status launch_wait_timeout(int* status, uint64_t limit_ns, cudaStream_t st) 
 
 size_t hkvd_ws_bytes(int64_t) { return 0; }
 
+kvb_status launch_deviation(const uint16_t* ka, int64_t lda, const uint16_t* kb, int64_t ldb, int64_t n, int kv_dim,
+                            float* dev, cudaStream_t st) {
+    int64_t blocks = (n + 7) / 8;
+    const int64_t cap = (int64_t)num_sms() * 16;
+    if (blocks > cap) blocks = cap;
+    dev_kernel<<<(unsigned)blocks, 256, 0, st>>>(ka, lda, kb, ldb, n, kv_dim, dev);
+    count_launch();
+    return cuda_ok(cudaGetLastError(), "deviation launch");
+}
+
 kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t* k_cached, int64_t ld_cached,
                        int64_t n_ctx, int kv_dim, int64_t k, int32_t* sel_out, float* dev_out, void*,
                        cudaStream_t st) {

@@ -96,6 +96,13 @@ kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t
                        cudaStream_t st);
 
 kvb_status launch_wait_timeout(int* status, uint64_t limit_ns, cudaStream_t st);
+kvb_status launch_deviation(const uint16_t* ka, int64_t lda, const uint16_t* kb, int64_t ldb, int64_t n, int kv_dim,
+                            float* dev, cudaStream_t st);
+kvb_status launch_window_select(const int32_t* win_start, int32_t n_win, int32_t window, int64_t n_ctx,
+                                uint8_t* flags, int32_t* sel, int64_t* k_out, cudaStream_t st);
+kvb_status launch_deviation_histogram(const uint16_t* ka, int64_t lda, const uint16_t* kb, int64_t ldb, int64_t n,
+                                      int kv_dim, const float* edges, int n_edges, float* dev,
+                                      unsigned long long* hist, cudaStream_t st);
 kvb_status launch_lmhead(const uint16_t* W, int64_t vocab, int H, const float* x, int n, float* logits,
                          unsigned long long* keys, int32_t* tokens, cudaStream_t st);
 

@@ -97,6 +97,10 @@ _SIGS = {
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
     "kvb_debug_wait_timeout": (c_i32, [c_vp, c_sz, c_i64, c_vp]),
     "kvb_lm_head_argmax": (c_i32, [P(Config), c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_sz, c_vp]),
+    "kvb_window_select_workspace_size": (c_sz, [c_i64]),
+    "kvb_window_select": (c_i32, [c_vp, c_i32, c_i32, c_i64, c_vp, c_vp, c_vp, c_sz, c_vp]),
+    "kvb_key_deviation_histogram": (c_i32, [c_vp, c_i64, c_vp, c_i64, c_i64, c_i32, c_vp, c_i32, c_vp, c_vp, c_vp,
+                                            c_sz, c_vp]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -225,6 +229,49 @@ def lm_head_argmax(cfg: Config, lm_head: torch.Tensor, hidden: torch.Tensor, log
           _ptr(hidden, torch.float32, "hidden"), n, _ptr(logits, torch.float32, "logits"),
           _ptr(tokens, torch.int32, "tokens"), _ptr(ws), ws.numel(), _stream())
     return tokens, logits
+
+
+def window_select(win_start: torch.Tensor, window: int, n_ctx: int, sel_out: Optional[torch.Tensor] = None,
+                  ws: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, int]:
+    """EPIC / KVLink selection: the union of [s, s + window) over the window starts, cut to
+    the context, ascending.  Returns (the selection, its length); reading the length waits
+    for the stream."""
+    dev = win_start.device
+    n_win = win_start.numel()
+    if sel_out is None:
+        sel_out = torch.empty(max(min(n_ctx, n_win * window), 1), dtype=torch.int32, device=dev)
+    need = lib().kvb_window_select_workspace_size(n_ctx)
+    if ws is None:
+        ws = torch.zeros(need, dtype=torch.uint8, device=dev)
+    k_out = torch.zeros(1, dtype=torch.int64, device=dev)
+    _call("kvb_window_select", _ptr(win_start, torch.int32, "win_start"), n_win, window, n_ctx,
+          _ptr(sel_out, torch.int32, "sel_out"), _ptr(k_out, torch.int64, "k_out"), _ptr(ws), ws.numel(), _stream())
+    k = int(k_out.item())
+    return sel_out[:k], k
+
+
+def key_deviation_histogram(k_a: torch.Tensor, k_b: torch.Tensor, edges: torch.Tensor,
+                            dev_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Per-token squared key difference between two [n][kv_dim] bf16 key sets (row strides
+    taken from the tensors), binned by `edges`; returns int64 counts [len(edges) + 1]."""
+    n = k_a.shape[0]
+    kv_dim = k_a[0].numel() if n else k_a.shape[-1]
+    if k_b.shape[0] != n:
+        raise ValueError("k_a and k_b need the same number of rows")
+    for t, nm in ((k_a, "k_a"), (k_b, "k_b")):
+        if t.dtype != torch.bfloat16 or not t.is_cuda:
+            raise ValueError(f"{nm} must be a CUDA bf16 tensor")
+        if n and not t[0].is_contiguous():
+            raise ValueError(f"{nm} rows must be contiguous")
+    ld_a = k_a.stride(0)
+    ld_b = k_b.stride(0)
+    hist = torch.empty(edges.numel() + 1, dtype=torch.int64, device=k_a.device)
+    if ws is None:
+        ws = torch.zeros(256 + (0 if dev_out is not None else 4 * n + 16), dtype=torch.uint8, device=k_a.device)
+    _call("kvb_key_deviation_histogram", k_a.data_ptr(), ld_a, k_b.data_ptr(), ld_b, n, kv_dim,
+          _ptr(edges, torch.float32, "edges"), edges.numel(), _ptr(dev_out, torch.float32, "dev_out"),
+          _ptr(hist, torch.int64, "hist"), _ptr(ws), ws.numel(), _stream())
+    return hist
 
 
 def debug_wait_timeout(ws: torch.Tensor, limit_ns: int) -> None:

@@ -13,7 +13,9 @@ followed by the question):
 * embedding table: N(0, 1), rounded to bf16;
 * linear weights: N(0, 0.02), rounded to bf16 (so both sides read the same values);
 * RMSNorm gains: 1.0;
-* chunks of equal length laid end to end, then a query suffix.
+* chunks of equal length laid end to end, then a query suffix;
+* optionally two special tokens between consecutive documents (the last two ids of
+  the vocabulary), whose rows of the concatenated cache are zero.
 
 Every tensor is drawn from its own generator, seeded from (seed, layer, name), so
 one layer can be regenerated without drawing the others.
@@ -28,7 +30,7 @@ import torch
 __all__ = [
     "ModelShape", "Workload", "SHAPES", "WORKLOADS", "tensor_seed",
     "make_layer_weights", "make_embed", "make_lm_head", "make_model", "make_tokens",
-    "chunk_starts_equal", "randn_bf16",
+    "chunk_starts_equal", "separator_layout", "separator_ids", "randn_bf16",
 ]
 
 
@@ -68,7 +70,10 @@ class ModelShape:
 
 @dataclasses.dataclass(frozen=True)
 class Workload:
-    """A request: `n_chunks` chunks of `chunk_len` tokens, a query suffix, ratio r."""
+    """A request: `n_chunks` chunks of `chunk_len` tokens, a query suffix, ratio r.
+
+    With n_sep > 0, n_sep special tokens sit between consecutive chunks (documents);
+    their cache rows are zero in the concatenated cache."""
     name: str
     shape: ModelShape
     n_chunks: int
@@ -76,17 +81,35 @@ class Workload:
     n_query: int
     r: float = 0.15
     check_layer: int = 1
+    n_sep: int = 0
 
     @property
     def n_ctx(self) -> int:
-        return self.n_chunks * self.chunk_len
+        return self.n_chunks * self.chunk_len + max(self.n_chunks - 1, 0) * self.n_sep
 
     @property
     def n_total(self) -> int:
         return self.n_ctx + self.n_query
 
     def chunk_starts(self) -> List[int]:
-        return chunk_starts_equal(self.n_chunks, self.chunk_len)
+        """Boundaries of every segment of the context (documents and separator groups), then n_ctx."""
+        return separator_layout(self.n_chunks, self.chunk_len, self.n_sep)[0]
+
+    def sep_starts(self) -> List[int]:
+        """First row of each separator group."""
+        return separator_layout(self.n_chunks, self.chunk_len, self.n_sep)[1]
+
+    def sep_rows(self) -> List[int]:
+        return [s + j for s in self.sep_starts() for j in range(self.n_sep)]
+
+    def tokens(self, seed: int = 1, device: str | torch.device = "cpu") -> torch.Tensor:
+        """Uniform token ids, with the separator ids at the separator rows."""
+        t = make_tokens(self.shape, self.n_total, seed)
+        ids = separator_ids(self.shape, self.n_sep)
+        for s in self.sep_starts():
+            for j, tok in enumerate(ids):
+                t[s + j] = tok
+        return t.to(device)
 
 
 TINY = ModelShape(hidden=256, n_q_heads=4, n_kv_heads=2, head_dim=64, mlp_dim=688,
@@ -104,6 +127,10 @@ WORKLOADS: Dict[str, Workload] = {
     "l8b_1layer": Workload("llama8b-2L-8x480+64", LLAMA8B.with_layers(2), 8, 480, 64),
     "l8b_32k": Workload("llama8b-32L-64x512+128", LLAMA8B, 64, 512, 128),
     "l8b_124k": Workload("llama8b-32L-242x512+128", LLAMA8B, 242, 512, 128),
+    # two special tokens between documents, their cache rows zero
+    "tiny_sep": Workload("tiny-2L-4x126+sep2+32", TINY, 4, 126, 32, n_sep=2),
+    "l8b_1layer_sep": Workload("llama8b-2L-8x478+sep2+64", LLAMA8B.with_layers(2), 8, 478, 64, n_sep=2),
+    "l8b_124k_sep": Workload("llama8b-32L-242x512+sep2+128", LLAMA8B, 242, 512, 128, n_sep=2),
 }
 
 
@@ -175,4 +202,23 @@ def make_tokens(shape: ModelShape, n: int, seed: int = 1, device: str | torch.de
 
 def chunk_starts_equal(n_chunks: int, chunk_len: int) -> List[int]:
     return [c * chunk_len for c in range(n_chunks + 1)]
+
+
+def separator_layout(n_chunks: int, chunk_len: int, n_sep: int):
+    """Documents of chunk_len tokens with n_sep special tokens between consecutive ones.
+    Returns (segment boundaries ending with n_ctx, first row of each separator group)."""
+    starts, seps, pos = [0], [], 0
+    for c in range(n_chunks):
+        pos += chunk_len
+        starts.append(pos)
+        if c + 1 < n_chunks and n_sep > 0:
+            seps.append(pos)
+            pos += n_sep
+            starts.append(pos)
+    return starts, seps
+
+
+def separator_ids(shape: ModelShape, n_sep: int) -> List[int]:
+    """Token ids of the special separator tokens: the last n_sep ids of the vocabulary."""
+    return [shape.vocab - n_sep + j for j in range(n_sep)]
 

@@ -317,3 +317,39 @@ def test_lm_head_argmax_rejects_bad_arguments(kvb):
     with pytest.raises(kvb.KvbError):
         kvb.lm_head_argmax(cfg, w, torch.zeros(1, 256, device="cuda"),
                            ws=torch.zeros(64, dtype=torch.uint8, device="cuda"))
+
+
+# ---------------------------------------------------------------- EPIC / KVLink windows, deviation histogram
+
+@pytest.mark.parametrize("starts,window,n_ctx", [
+    (synth.WORKLOADS["l8b_124k_sep"].sep_starts(), 20, synth.WORKLOADS["l8b_124k_sep"].n_ctx),   # EPIC, 124k
+    (synth.WORKLOADS["l8b_124k_sep"].sep_starts(), 2, synth.WORKLOADS["l8b_124k_sep"].n_ctx),    # KVLink
+    ([5, 3, 40, -7, 97, 1000, 99], 20, 100),       # overlapping, unsorted, outside the context
+    ([], 20, 100),
+    ([0, 10], 0, 100),
+    ([0], 50000, 40000),                             # one window covering everything
+])
+def test_window_select_bit_exact(kvb, starts, window, n_ctx):
+    sel, k = kvb.window_select(torch.tensor(starts, dtype=torch.int32, device="cuda"), window, n_ctx)
+    want = blend.window_select(starts, window, n_ctx)
+    assert k == len(want) and np.array_equal(sel.cpu().numpy(), want)
+
+
+@pytest.mark.parametrize("n,kv_dim,ld", [(123904, 1024, 1024), (1000, 128, 256), (1, 8, 8), (0, 1024, 1024)])
+def test_key_deviation_histogram(kvb, n, kv_dim, ld):
+    a = synth.randn_bf16((max(n, 1), ld), 601)[:n]
+    b = (a.float() + synth.randn_bf16((max(n, 1), ld), 602, 0.05)[:n].float()
+         * torch.rand(max(n, 1), 1, generator=torch.Generator().manual_seed(3))[:n] ** 4).to(torch.bfloat16)
+    b[: n // 3] = a[: n // 3]                        # exact zeros
+    edges = torch.tensor([0.0] + [10.0 ** e for e in np.arange(-8, 3.01, 0.25)], dtype=torch.float32)
+    da, db = dev(a), dev(b)
+    d = torch.empty(max(n, 1), dtype=torch.float32, device="cuda")
+    h = kvb.key_deviation_histogram(da[:, :kv_dim], db[:, :kv_dim], dev(edges), dev_out=d[:n] if n else None)
+    h2 = kvb.key_deviation_histogram(da[:, :kv_dim], db[:, :kv_dim], dev(edges))   # deviation in the workspace
+    torch.cuda.synchronize()
+    got = d[:n].cpu().numpy()
+    want = blend.hkvd_deviation(np64(a[:, :kv_dim]), np64(b[:, :kv_dim]))
+    # fp32 sum of kv_dim exact squares of bf16 differences: relative bound kv_dim * 2^-24 (+ the square)
+    assert np.all(np.abs(got - want) <= (kv_dim + 2) * 2.0 ** -24 * want)
+    assert np.array_equal(h.cpu().numpy(), blend.deviation_histogram(got, edges.numpy()))
+    assert torch.equal(h, h2) and int(h.sum()) == n

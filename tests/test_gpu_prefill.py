@@ -38,12 +38,16 @@ class Case:
         self.n_ctx, self.nq, self.N = wl.n_ctx, wl.n_query, wl.n_total
         w = synth.make_model(self.shape, 0)
         self.w = w
-        self.toks = synth.make_tokens(self.shape, self.N, 1)
+        self.toks = wl.tokens()
+        self.sep_rows = wl.sep_rows()
         self.s = Shape.of(self.shape, act_bf16=True)
         self.s64 = Shape.of(self.shape)
         self.l64 = [{k: llama.as64(v) for k, v in l.items()} for l in w["layers"]]
         x0 = blend.embed_rows(w["embed"], self.toks.numpy())
         self.cc = blend.chunk_caches(self.s, self.l64, x0[: self.n_ctx], self.starts)
+        if self.sep_rows:
+            self.cc = blend.zero_kv_rows(self.cc, self.sep_rows)
+        self.x0 = x0
         self.sel = blend.selective_prefill(self.s, self.l64, x0, self.starts, self.nq, wl.r, self.cc["k"],
                                            self.cc["v"], 1, None, w["final_norm"])
         self.full = blend.full_prefill(self.s, self.l64, x0)
@@ -99,7 +103,7 @@ class Case:
 _CASES = {}
 
 
-@pytest.fixture(scope="module", params=["tiny", "l8b_1layer"])
+@pytest.fixture(scope="module", params=["tiny", "l8b_1layer", "tiny_sep", "l8b_1layer_sep"])
 def case(request, kvb):
     if request.param not in _CASES:
         _CASES[request.param] = Case(kvb, synth.WORKLOADS[request.param])
@@ -120,7 +124,8 @@ def test_full_prefill_matches_oracle(kvb, case):
 
 
 def test_chunk_caches_match_oracle(kvb, case):
-    k, v = workload.chunk_caches(case.cfg, case.model, case.rope, case.dtoks[: case.n_ctx], case.starts, ws=case.ws)
+    k, v = workload.chunk_caches(case.cfg, case.model, case.rope, case.dtoks[: case.n_ctx], case.starts, ws=case.ws,
+                                 zero_rows=case.sep_rows)
     torch.cuda.synchronize()
     assert kvb.device_status(case.ws) == 0
     for l in range(case.shape.n_layers):
@@ -226,3 +231,90 @@ def test_pipelined_host_ingest_equals_device_resident(kvb, case):
     with pytest.raises(ValueError):   # pageable memory is refused by the binding
         kvb.selective_prefill_host(case.cfg, case.model, case.rope, hk.clone(), hv, ck2, cv2, case.dtoks,
                                    case.dstarts, case.n_ctx, case.nq, case.wl.r, 1)
+
+
+def test_epic_and_kvlink_selection(kvb, case):
+    """Separator workloads: the EPIC set (20 rows from every separator) and the KVLink set
+    (the separators) built on the device equal the oracle's; the selective prefill with the
+    EPIC set matches the oracle; separator rows left out keep zero K/V in the selective layers."""
+    if not case.sep_rows:
+        pytest.skip("no separators in this workload")
+    seps = case.wl.sep_starts()
+    dseps = torch.tensor(seps, dtype=torch.int32, device="cuda")
+    for window in (20, case.wl.n_sep):
+        got, k = kvb.window_select(dseps, window, case.n_ctx)
+        assert np.array_equal(got.cpu().numpy(), blend.window_select(seps, window, case.n_ctx))
+    epic = blend.window_select(seps, 20, case.n_ctx)
+    ref = blend.selective_prefill(case.s, case.l64, case.x0, case.starts, case.nq, 0.0, case.cc["k"], case.cc["v"], 1,
+                                  epic, case.w["final_norm"])
+    ck, cv = case.new_cache()
+    sel_dev, _ = kvb.window_select(dseps, 20, case.n_ctx)
+    fh, sel, _ = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks,
+                                       case.dstarts, case.n_ctx, case.nq, 0.0, 1, forced_sel=sel_dev, ws=case.ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(case.ws) == 0
+    e = case.check_fh(fh.cpu(), ref["final_hidden"], "final hidden (EPIC selection)")
+    for l in range(1, case.shape.n_layers):
+        case.check_cache(ck[l].cpu(), ref["k"][l], f"k{l}", f"EPIC blended K layer {l}")
+    # KVLink's set recomputes exactly the separators; any other set leaves them zero
+    one = torch.tensor([case.sep_rows[-1] + case.wl.n_sep], dtype=torch.int32, device="cuda")
+    ck, cv = case.new_cache()
+    kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks, case.dstarts,
+                          case.n_ctx, case.nq, 0.0, 1, forced_sel=one, ws=case.ws)
+    torch.cuda.synchronize()
+    rows = torch.tensor(case.sep_rows, device="cuda")
+    assert torch.all(ck[1:, rows] == 0) and torch.all(cv[1:, rows] == 0)
+    assert torch.all(ck[0, rows].abs().sum(dim=(-1, -2)) > 0)          # layer 0 is recomputed in full
+    print("EPIC", case.wl.name, len(epic), "rows", e)
+
+
+def test_key_deviation_histogram_at_check_layer(kvb, case):
+    """Distribution of squared key differences against the full prefill at the check layer:
+    plain concatenation (r = 0) gives the deviations HKVD ranks (bit-equal to the ones it
+    ranked); the r = 0.15 blend zeroes exactly its k rows, which are the k largest; EPIC
+    zeroes its windows.  Counts are exact against the oracle's binning of the same values."""
+    nc = case.n_ctx
+    ckf, cvf = case.new_cache()
+    kvb.full_prefill(case.cfg, case.model, case.rope, ckf, cvf, case.dtoks, n_out=case.nq, ws=case.ws)
+    kd = case.shape.kv_dim
+
+    def blend_cache(r, forced=None):
+        ck, cv = case.new_cache()
+        _, sel, _ = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks,
+                                          case.dstarts, nc, case.nq, r, 1, forced_sel=forced, ws=case.ws)
+        return ck, sel
+
+    edges = torch.tensor([0.0] + [10.0 ** e for e in np.arange(-6, 3.01, 0.5)], dtype=torch.float32, device="cuda")
+    ed = edges.cpu().numpy()
+
+    def dev_hist(ck):
+        dev = torch.empty(nc, dtype=torch.float32, device="cuda")
+        h = kvb.key_deviation_histogram(ck[1, :nc].view(nc, kd), ckf[1, :nc].view(nc, kd), edges, dev_out=dev)
+        torch.cuda.synchronize()
+        d = dev.cpu().numpy()
+        assert np.array_equal(h.cpu().numpy(), blend.deviation_histogram(d, ed))
+        return d, h.cpu().numpy()
+
+    ck0, _ = blend_cache(0.0)
+    d0, h0 = dev_hist(ck0)
+    ref = blend.hkvd_deviation(np64(ck0[1, :nc].cpu()), np64(ckf[1, :nc].cpu()))
+    assert np.allclose(d0, ref, rtol=1e-5, atol=1e-30)
+    k = blend.num_selected(case.wl.r, nc)
+    cks, sel = blend_cache(case.wl.r)
+    s = sel[:k].cpu().numpy().astype(np.int64)
+    assert np.array_equal(s, blend.topk_select(d0, k))          # HKVD ranked these very values
+    ds, hs = dev_hist(cks)
+    want = d0.copy()
+    want[s] = 0.0
+    assert np.array_equal(ds, want)
+    assert hs.sum() == nc
+    if 0 < k < nc:
+        assert ds.max() <= np.sort(d0)[-k - 1]                    # the k largest deviations are gone
+    epic = blend.window_select(case.wl.sep_starts(), 20, nc)
+    if len(epic):
+        cke, _ = blend_cache(0.0, torch.from_numpy(epic.astype(np.int32)).cuda())
+        de, _ = dev_hist(cke)
+        want = d0.copy()
+        want[epic] = 0.0
+        assert np.array_equal(de, want)
+    print("check-layer deviation", case.wl.name, "r=0", h0.tolist(), "hkvd", hs.tolist())

@@ -455,3 +455,75 @@ def test_first_token_is_argmax_with_lowest_id_on_ties():
     for r in range(3):
         best = max(range(50), key=lambda v: (sum(h[r, d] * w[v, d] for d in range(16)), -v))
         assert tok[r] == best
+
+
+# ------------------------------------------------------------------ separators, EPIC, deviation histogram
+
+def test_separator_layout_and_tokens():
+    from paper_2609_09768_gb300 import synth
+    starts, seps = synth.separator_layout(3, 5, 2)
+    assert starts == [0, 5, 7, 12, 14, 19] and seps == [5, 12]
+    wl = synth.WORKLOADS["tiny_sep"]
+    t = wl.tokens()
+    assert len(t) == wl.n_total and wl.n_ctx == 4 * 126 + 3 * 2
+    for s in wl.sep_starts():
+        assert [int(t[s]), int(t[s + 1])] == [wl.shape.vocab - 2, wl.shape.vocab - 1]
+
+
+def test_window_select_epic_and_kvlink():
+    # EPIC: 20 rows from every separator start; windows overlap and run past the context end
+    assert list(blend.window_select([3, 10], 20, 25)) == list(range(3, 25))
+    assert list(blend.window_select([5, 12], 2, 19)) == [5, 6, 12, 13]              # KVLink: the separators
+    assert list(blend.window_select([], 20, 10)) == []
+    assert list(blend.window_select([9], 20, 10)) == [9]
+    assert list(blend.window_select([4, 0], 3, 10)) == [0, 1, 2, 4, 5, 6]          # order of starts is free
+    # closed form for disjoint windows inside the context
+    sel = blend.window_select([100 * c for c in range(1, 9)], 20, 1000)
+    assert len(sel) == 8 * 20 and np.all(np.diff(sel) > 0)
+
+
+def test_zero_separator_rows_stay_zero_after_realign():
+    s = Shape(hidden=16, n_q_heads=2, n_kv_heads=1, head_dim=8, mlp_dim=24, rms_eps=1e-5, rope_theta=1e4)
+    rng = np.random.default_rng(3)
+    cc = {"k": rng.standard_normal((2, 12, 1, 8)), "v": rng.standard_normal((2, 12, 1, 8))}
+    z = blend.zero_kv_rows(cc, [5, 6])
+    assert np.all(z["k"][:, [5, 6]] == 0) and np.all(z["v"][:, [5, 6]] == 0)
+    assert np.array_equal(z["k"][:, :5], cc["k"][:, :5]) and np.array_equal(z["v"][:, 7:], cc["v"][:, 7:])
+    r = blend.realign(s, z["k"], [0, 5, 7, 12])
+    assert np.all(r[:, [5, 6]] == 0)
+
+
+def test_deviation_histogram_bins():
+    edges = np.array([1e-3, 1e-2, 1e-1, 1.0])
+    dev = np.array([0.0, 1e-3, 5e-3, 1e-2, 0.5, 1.0, 7.0, 9e-4])
+    assert list(blend.deviation_histogram(dev, edges)) == [2, 2, 1, 1, 2]
+    rng = np.random.default_rng(4)
+    d = rng.exponential(size=500)
+    e = np.sort(rng.exponential(size=7))
+    h = blend.deviation_histogram(d, e)
+    assert h.sum() == 500
+    assert np.array_equal(h, np.bincount(np.searchsorted(e, d, side="right"), minlength=8))
+
+
+def test_selective_prefill_with_separators_recompute_all_equals_full():
+    """r = 1 over a context with zeroed separator rows is still the full causal prefill:
+    every context row, separators included, is recomputed before it is read."""
+    s = Shape(hidden=16, n_q_heads=2, n_kv_heads=1, head_dim=8, mlp_dim=24, rms_eps=1e-5, rope_theta=1e4)
+    rng = np.random.default_rng(8)
+    layers = [{"attn_norm": np.ones(16), "mlp_norm": np.ones(16),
+               "w_qkv": rng.standard_normal((32, 16)) * 0.2, "w_o": rng.standard_normal((16, 16)) * 0.2,
+               "w_gate": rng.standard_normal((24, 16)) * 0.2, "w_up": rng.standard_normal((24, 16)) * 0.2,
+               "w_down": rng.standard_normal((16, 24)) * 0.2} for _ in range(3)]
+    starts, seps = [0, 5, 7, 12, 14, 19], [5, 12]
+    x0 = rng.standard_normal((23, 16))
+    cc = blend.zero_kv_rows(blend.chunk_caches(s, layers, x0[:19], starts), [5, 6, 12, 13])
+    full = blend.full_prefill(s, layers, x0)
+    sp = blend.selective_prefill(s, layers, x0, starts, 4, 1.0, cc["k"], cc["v"])
+    assert np.array_equal(sp["layer_out"][-1][-4:], full["x"][-4:])
+    # EPIC's rows are a valid forced selection; the separator rows it leaves out keep zero K/V
+    epic = blend.window_select(seps, 3, 19)
+    sp = blend.selective_prefill(s, layers, x0, starts, 4, 0.0, cc["k"], cc["v"], forced_sel=epic)
+    assert list(sp["sel"]) == [5, 6, 7, 12, 13, 14]
+    assert np.all(sp["k"][1:, [5, 6, 12, 13]] != 0)           # recomputed in the selective layers
+    kv = blend.selective_prefill(s, layers, x0, starts, 4, 0.0, cc["k"], cc["v"], forced_sel=[7])
+    assert np.all(kv["k"][1:, [5, 6, 12, 13]] == 0) and np.all(kv["v"][1:, [5, 6, 12, 13]] == 0)
