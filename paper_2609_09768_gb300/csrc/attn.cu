@@ -249,20 +249,24 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
 
             const int key0 = (t_begin + j) * KT_ROWS;
             const bool full_vis = key0 >= lo_max && key0 + KT_ROWS - 1 <= hi_min;
-            float mt = -INFINITY;
-            if (full_vis) {
-#pragma unroll
-                for (int c = 0; c < KT_ROWS; ++c) mt = fmaxf(mt, __uint_as_float(s[c]));
-            } else {
+            if (!full_vis) {
 #pragma unroll
                 for (int c = 0; c < KT_ROWS; ++c) {
                     const int key = key0 + c;
-                    float v = __uint_as_float(s[c]);
-                    if (key > hi || key < lo) v = -INFINITY;
-                    s[c] = __float_as_uint(v);
-                    mt = fmaxf(mt, v);
+                    if (key > hi || key < lo) s[c] = __float_as_uint(-INFINITY);
                 }
             }
+            // row max as a tree: 16 independent chains, not one 128-long dependent chain
+            float mx[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) mx[c] = __uint_as_float(s[c]);
+#pragma unroll
+            for (int c = 16; c < KT_ROWS; ++c) mx[c & 15] = fmaxf(mx[c & 15], __uint_as_float(s[c]));
+#pragma unroll
+            for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                for (int c = 0; c < w; ++c) mx[c] = fmaxf(mx[c], mx[c + w]);
+            const float mt = mx[0];
             const float m_new = fmaxf(m_run, mt);
             const bool resc = (m_new - m_run) * sl2 > RESCALE_LOG2;   // false when both are -inf
             float alpha = 1.f;
@@ -273,15 +277,15 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             }
             const float mref = ((m_run == -INFINITY) ? 0.f : m_run * sl2) - P_SHIFT_LOG2;
             uint32_t pk[KT_ROWS / 2];
-            float lsum = 0.f;
+            float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int c = 0; c < KT_ROWS; c += 2) {
                 const float e0 = fast_exp2(fmaf(__uint_as_float(s[c]), sl2, -mref));
                 const float e1 = fast_exp2(fmaf(__uint_as_float(s[c + 1]), sl2, -mref));
-                lsum += e0 + e1;
+                ls[(c >> 1) & 3] += e0 + e1;
                 pk[c / 2] = pack_f16(e0, e1);
             }
-            l_run += lsum;
+            l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
 
             if (j >= 1) {
                 if (!mbar_wait_warp(pv_done, (j - 1) & 1, abort_flag, p.status)) { ok = false; break; }
