@@ -14,7 +14,8 @@
 // TMEM columns: S double buffer [0, 256), O [256, 384), Q [384, 448), P [448, 512).
 //
 // Pipeline per key tile j (128 keys):
-//   TMA warp   : K_j, V_j into 3-deep rings (128-byte swizzle)
+//   TMA warp   : K_j and V_j together into a 3-deep ring (128-byte swizzle); slot
+//                j % 3 is reused once P.V of the tile that held it has completed
 //   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=128, K=16 steps,
 //                A = Q from TMEM); after the softmax of tile j-1,
 //                O += P_{j-1} V_{j-1} (A = P from TMEM, V an MN-major operand)
@@ -62,16 +63,17 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
+    // Every wait of the MMA thread and every tcgen05.commit costs the tensor pipe tens to
+    // hundreds of cycles, so each 128-key tile uses two of each: kv_full (K_j and V_j
+    // landed) and p_full (P_{j-1} written) for the MMA thread; s_full (S_j done) and
+    // pv_done (P.V_i done) as commits.  P.V_i done also frees slot i % STAGES for the
+    // producer (P_i was written after S_i had been read) and lets the softmax overwrite P.
     uint64_t* q_ready = bars + 0;                // Q rows stored into TMEM (4 warps)
-    uint64_t* k_full = bars + 1;                 // [STAGES]
-    uint64_t* k_empty = k_full + STAGES;         // [STAGES]
-    uint64_t* v_full = k_empty + STAGES;         // [STAGES]
-    uint64_t* v_empty = v_full + STAGES;         // [STAGES]
-    uint64_t* s_full = v_empty + STAGES;         // [2]
-    uint64_t* s_free = s_full + 2;               // [2]
-    uint64_t* p_full = s_free + 2;
-    uint64_t* pv_done = p_full + 1;
-    uint64_t* drain = pv_done + 1;
+    uint64_t* kv_full = bars + 1;                // [STAGES]: K_j and V_j in slot j % STAGES
+    uint64_t* s_full = kv_full + STAGES;         // [2]: S_j done, phase j/2 of s_full[j % 2]
+    uint64_t* p_full = s_full + 2;               // [STAGES]: P_j written, phase j/3 of p_full[j % 3]
+    uint64_t* pv_done = p_full + STAGES;         // [STAGES]: P.V_i done, phase i/3 of pv_done[i % 3]
+    uint64_t* drain = pv_done + STAGES;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* red = reinterpret_cast<int*>(tmem_slot + 2);   // lo_min, hi_max, hi_min, lo_max
@@ -86,12 +88,11 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     if (threadIdx.x == 0) {
         mbar_init(q_ready, 4);
         for (int st = 0; st < STAGES; ++st) {
-            mbar_init(&k_full[st], 1); mbar_init(&k_empty[st], 1);
-            mbar_init(&v_full[st], 1); mbar_init(&v_empty[st], 1);
+            mbar_init(&kv_full[st], 1);
+            mbar_init(&p_full[st], 4);
+            mbar_init(&pv_done[st], 1);
         }
-        for (int b = 0; b < 2; ++b) { mbar_init(&s_full[b], 1); mbar_init(&s_free[b], 4); }
-        mbar_init(p_full, 4);
-        mbar_init(pv_done, 1);
+        for (int b = 0; b < 2; ++b) mbar_init(&s_full[b], 1);
         mbar_init(drain, 1);
         *abort_flag = 0;
         red[0] = INT_MAX; red[1] = -1; red[2] = INT_MAX; red[3] = -1;
@@ -135,28 +136,21 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                 const int st = j % STAGES;
                 const uint32_t ph = (uint32_t)(j / STAGES) & 1;
                 const int y = (t_begin + j) * KT_ROWS;
-                if (!mbar_wait(&k_empty[st], ph ^ 1, abort_flag, p.status)) break;
-                mbar_expect_tx(&k_full[st], S::KV_BYTES);
+                // slot st is free once P.V_{j-STAGES} is done (its S had been read before P was written)
+                if (!mbar_wait(&pv_done[st], ph ^ 1, abort_flag, p.status)) break;
+                mbar_expect_tx(&kv_full[st], 2 * S::KV_BYTES);
 #pragma unroll
-                for (int c = 0; c < D / 64; ++c)
-                    tma_load_2d(sK + st * S::KV_BYTES + c * S::CHUNK, &tmK, &k_full[st], g * D + c * 64, y);
-                if (!mbar_wait(&v_empty[st], ph ^ 1, abort_flag, p.status)) { issued = -(j + 1); break; }
-                mbar_expect_tx(&v_full[st], S::KV_BYTES);
-#pragma unroll
-                for (int c = 0; c < D / 64; ++c)
-                    tma_load_2d(sV + st * S::KV_BYTES + c * S::CHUNK, &tmV, &v_full[st], g * D + c * 64, y);
+                for (int c = 0; c < D / 64; ++c) {
+                    tma_load_2d(sK + st * S::KV_BYTES + c * S::CHUNK, &tmK, &kv_full[st], g * D + c * 64, y);
+                    tma_load_2d(sV + st * S::KV_BYTES + c * S::CHUNK, &tmV, &kv_full[st], g * D + c * 64, y);
+                }
                 issued = j + 1;
             }
             // on the abort path, let the loads already issued land before exiting
             if (*abort_flag) {
-                const int nk = issued < 0 ? -issued : issued;      // K tiles issued
-                const int nv = issued < 0 ? -issued - 1 : issued;  // V tiles issued
                 const uint64_t t0 = globaltimer();
-                for (int j = (nk > STAGES ? nk - STAGES : 0); j < nk; ++j)
-                    while (!mbar_try_wait(&k_full[j % STAGES], (uint32_t)(j / STAGES) & 1) &&
-                           globaltimer() - t0 < 1000000ull) {}
-                for (int j = (nv > STAGES ? nv - STAGES : 0); j < nv; ++j)
-                    while (!mbar_try_wait(&v_full[j % STAGES], (uint32_t)(j / STAGES) & 1) &&
+                for (int j = (issued > STAGES ? issued - STAGES : 0); j < issued; ++j)
+                    while (!mbar_try_wait(&kv_full[j % STAGES], (uint32_t)(j / STAGES) & 1) &&
                            globaltimer() - t0 < 1000000ull) {}
             }
         }
@@ -171,8 +165,9 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             for (int j = 0; ok && j <= n_tiles; ++j) {
                 if (j < n_tiles) {
                     const int b = j & 1, st = j % STAGES;
-                    if (!mbar_wait(&k_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status)) break;
-                    if (j >= 2 && !mbar_wait(&s_free[b], ((j - 2) >> 1) & 1, abort_flag, p.status)) break;
+                    // S buffer b last held S_{j-2}: the softmax read it before writing P_{j-2},
+                    // which this thread waited for in the previous iteration
+                    if (!mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
                     // descriptor built once per tile; constant steps inside the unrolled loop keep
                     // the issuing thread ahead of the 64-cycle MMAs
@@ -184,13 +179,12 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                         mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32), IDESC_S,
                                    kk > 0 ? 1u : 0u);
                     }
-                    mma_commit(&k_empty[st]);
                     mma_commit(&s_full[b]);
                 }
                 if (j >= 1) {
                     const int i = j - 1, st = i % STAGES;
-                    if (!mbar_wait(p_full, i & 1, abort_flag, p.status)) break;
-                    if (!mbar_wait(&v_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
+                    // V_i landed with K_i (kv_full waited in iteration i)
+                    if (!mbar_wait(&p_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
                     const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
                     const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_P;
@@ -200,8 +194,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                         // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
                         mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
                     }
-                    mma_commit(&v_empty[st]);
-                    mma_commit(pv_done);
+                    mma_commit(&pv_done[st]);
                 }
             }
             mma_commit(drain);
@@ -243,9 +236,6 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
 #pragma unroll
             for (int c = 0; c < KT_ROWS / 32; ++c) tmem_ld32(tmem_base + lane_addr + b * KT_ROWS + c * 32, s + c * 32);
             tmem_ld_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_free[b]);
 
             const int key0 = (t_begin + j) * KT_ROWS;
             const bool full_vis = key0 >= lo_max && key0 + KT_ROWS - 1 <= hi_min;
@@ -288,7 +278,11 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
 
             if (j >= 1) {
-                if (!mbar_wait_warp(pv_done, (j - 1) & 1, abort_flag, p.status)) { ok = false; break; }
+                if (!mbar_wait_warp(&pv_done[(j - 1) % STAGES], (uint32_t)((j - 1) / STAGES) & 1, abort_flag,
+                                    p.status)) {
+                    ok = false;
+                    break;
+                }
                 tc_fence_after();
                 if (__any_sync(0xffffffffu, resc)) {
                     const uint32_t oaddr = tmem_base + lane_addr + COL_O;
@@ -310,9 +304,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(p_full);
+            if (lane == 0) mbar_arrive(&p_full[j % STAGES]);
         }
-        if (ok && mbar_wait_warp(pv_done, (n_tiles - 1) & 1, abort_flag, p.status)) {
+        if (ok && mbar_wait_warp(&pv_done[(n_tiles - 1) % STAGES], (uint32_t)((n_tiles - 1) / STAGES) & 1, abort_flag,
+                                 p.status)) {
             tc_fence_after();
             const uint32_t oaddr = tmem_base + lane_addr + COL_O;
             const float inv = (l_run > 0.f) ? 1.f / l_run : 0.f;
