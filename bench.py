@@ -37,7 +37,7 @@ METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % 
 # size (18,713 rows over a 124,032-row cache), from the ncu capture summarised in
 # profiles/attn_kernel_sparse_m18713_nkv124032.md; valid only for the kernel sources it
 # was taken on (sha1 prefixes of attn.cu and common.cuh), otherwise reported as null.
-ATTN_TRAFFIC = {"bytes": 8.167612e9 + 0.141560e9, "sha1": {"attn.cu": "6135d4e73a3c", "common.cuh": "1bea4aeef0d1"}}
+ATTN_TRAFFIC = {"bytes": 8.171074e9 + 0.141687e9, "sha1": {"attn.cu": "53c3e0fbf4ab", "common.cuh": "1bea4aeef0d1"}}
 
 
 def attn_traffic():
