@@ -60,6 +60,7 @@ def parse():
     ap.add_argument("--r", type=float, default=None)
     ap.add_argument("--r1-steps", type=int, default=1, help="timed steps of the r = 1.0 comparator (0: skip)")
     ap.add_argument("--e2e-steps", type=int, default=2, help="timed end-to-end steps (0: skip)")
+    ap.add_argument("--decode-steps", type=int, default=16, help="greedy decode steps timed after the prefill (0: skip)")
     ap.add_argument("--cpu-rows", type=int, default=512, help="rows in the oracle's timed sample")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--sweep", action="store_true",
@@ -216,13 +217,15 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     weights = workload.device_model(shape, seed=0, device=dev, draw_on_device=True)
     model = kvb.Model(weights)
     toks = synth.make_tokens(shape, N, 1).to(dev)
-    rope = kvb.RopeTable(cfg, N, dev)
+    n_dec = max(args.decode_steps, 0)
+    cap = N + n_dec + 1                      # cache rows: the prompt, then the decoded tokens
+    rope = kvb.RopeTable(cfg, cap, dev)
     ws = kvb.workspace(cfg, N, dev)
     starts = wl.chunk_starts()
     dstarts = torch.tensor(starts, dtype=torch.int32, device=dev)
     kch, vch = workload.chunk_caches(cfg, model, rope, toks[:n_ctx], starts, ws=ws)
-    ck = torch.empty(L, N, Hkv, D, dtype=torch.bfloat16, device=dev)
-    cv = torch.empty(L, N, Hkv, D, dtype=torch.float16, device=dev)
+    ck = torch.empty(L, cap, Hkv, D, dtype=torch.bfloat16, device=dev)
+    cv = torch.empty(L, cap, Hkv, D, dtype=torch.float16, device=dev)
     fh = torch.empty(nq, H, dtype=torch.float32, device=dev)
     sel = torch.empty(n_ctx, dtype=torch.int32, device=dev)
     lm = synth.make_lm_head(shape, 0, dev)
@@ -369,6 +372,63 @@ def run_ours(args, wl, rank: int, world: int) -> None:
                "bare_h2d_ms": round(h2d_ms, 2), "bare_h2d_gbs": round(h2d / (h2d_ms * 1e-3) / 1e9, 1)}
         del hk, hv, kd, wsp
 
+    # greedy decode after the prefill (first token already decoded by the step): n_dec steps
+    # through kvb_decode_step, position and tokens on the device; eager launches, then the
+    # same step replayed as a CUDA graph
+    decode = None
+    if n_dec > 0:
+        step()                                             # fresh prefill cache + first token
+        tokens = torch.zeros(cap + 1, dtype=torch.int32, device=dev)
+        tokens[:N] = toks
+        tokens[N:N + 1] = tok
+        pos = torch.tensor([N], dtype=torch.int32, device=dev)
+        dws = kvb.decode_workspace(cfg, cap, dev)
+        kvb.decode_step(cfg, model, rope, ck, cv, lm, tokens, pos, cap, ws=dws)   # warm-up (position N)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(n_dec - 1):
+            kvb.decode_step(cfg, model, rope, ck, cv, lm, tokens, pos, cap, ws=dws)
+        b.record()
+        torch.cuda.synchronize()
+        # embed; per layer 2 RMSNorms, 4 GEMVs, RoPE/append, attention + combine; final norm,
+        # lm_head + argmax, position/token update
+        launches = 1 + 9 * L + 1 + 2 + 1
+        dec_ms = a.elapsed_time(b) / max(n_dec - 1, 1)
+        assert kvb.device_status(dws) == 0 and int(pos.item()) == N + n_dec
+        p_mid = N + n_dec // 2
+        w_bytes = float(L * 2 * (shape.qkv_dim * H + H * shape.q_dim + 3 * H * F) + shape.vocab * H * 2)
+        kv_bytes = float(L * (p_mid + 1) * shape.kv_dim * 2 * 2)
+        graph_ms = None
+        try:
+            pos.fill_(N)
+            g = torch.cuda.CUDAGraph()
+            cs = torch.cuda.Stream(device=dev)
+            cs.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(cs):
+                with torch.cuda.graph(g, stream=cs):
+                    kvb.decode_step(cfg, model, rope, ck, cv, lm, tokens, pos, cap, ws=dws)
+            torch.cuda.current_stream().wait_stream(cs)
+            pos.fill_(N)
+            g.replay()
+            torch.cuda.synchronize()
+            a.record()
+            for _ in range(n_dec - 1):
+                g.replay()
+            b.record()
+            torch.cuda.synchronize()
+            assert kvb.device_status(dws) == 0 and int(pos.item()) == N + n_dec
+            graph_ms = a.elapsed_time(b) / max(n_dec - 1, 1)
+        except Exception as exc:                          # report the eager number alone
+            print(f"decode graph capture skipped: {exc}", file=sys.stderr)
+        best = min(dec_ms, graph_ms) if graph_ms else dec_ms
+        decode = {"tokens": n_dec, "positions": [N, N + n_dec], "ms_per_token": round(dec_ms, 4),
+                  "graph_ms_per_token": round(graph_ms, 4) if graph_ms else None,
+                  "bytes_per_token": w_bytes + kv_bytes, "weights_bytes": w_bytes, "kv_bytes": kv_bytes,
+                  "gbs": round((w_bytes + kv_bytes) / (best * 1e-3) / 1e9, 1),
+                  "frac_of_hbm": round((w_bytes + kv_bytes) / (best * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                  "launches_per_token": int(launches)}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         n = args.cpu_rows
@@ -397,7 +457,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
             "algorithmic_tflops": round(total_flop / (ms * 1e-3) / 1e12, 2),
             "stages_ms": stages, "kernels": dict(kdict, first_token_lm_head=lm_head),
             "first_token": int(tok.item()),
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "decode": decode,
             "gpu_launches": int(sum(t["n_launches"] for t in tims)) + 2 * args.steps,
             "clocks": clk,
         }

@@ -381,6 +381,40 @@ kvb_status kvb_key_deviation_histogram(const uint16_t* k_a, int64_t ld_a, const 
                                        int32_t kv_dim, const float* edges, int32_t n_edges, float* dev_out,
                                        int64_t* hist_out, void* ws, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------- greedy decode
+ * After the prefill, the paper generates with greedy decoding (Sec. 4): each step feeds
+ * the last token through every layer at the next position, appends its K/V to the
+ * cache and takes the argmax of the logits.  One step:
+ *   x = embed[tokens[p]];  for each layer: the decoder block of Sec. 4's model on the
+ *   single row at position p (RoPE at p; K/V written into cache row p; attention over
+ *   cache rows [0, p]);  tokens[p + 1] = argmax(RMSNorm(x) * lm_head^T) (ties to the
+ *   lower id);  p = p + 1.
+ * `pos` (int32 [1]) and `tokens` (int32, room for max_pos + 1 ids) live in device
+ * memory and are updated on the device, so consecutive steps need no host value; a
+ * step needs 0 <= *pos < max_pos, otherwise it records KVB_ERR_INVALID_ARG in the
+ * workspace status word (read with kvb_device_status) and writes nothing.
+ * cache: rows [0, *pos) hold the prompt's blended cache (the prefill's output), at
+ * least max_pos rows per layer; rope: at least max_pos positions; lm_head: bf16
+ * [vocab][H]; hidden_out: fp32 [H] final hidden state of the step, or NULL.
+ * Workspace: kvb_decode_workspace_size(cfg, max_pos) bytes (status word, activations,
+ * per-split attention partials).  Errors: INVALID_ARG, UNSUPPORTED (hidden, mlp_dim or
+ * Hq*D above 16384; head_dim 128 with 2, 4 or 8 q heads per kv head, or head_dim 64
+ * with 2 or 4), WORKSPACE. */
+kvb_status kvb_decode_workspace_size(const kvb_config* cfg, int64_t max_pos, size_t* bytes);
+kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
+                           const kvb_kv_cache* cache, const uint16_t* lm_head, int32_t* tokens, int32_t* pos,
+                           int64_t max_pos, float* hidden_out, void* ws, size_t ws_bytes, void* stream);
+
+/* The decode step's attention alone: the new row's q (bf16 [Hq][D], RoPE applied)
+ * over one layer's cache rows [0, *pos] (k_layer bf16, v_layer fp16 holding
+ * bf16-precision values, both [n_rows][Hkv][D], n_rows >= max_pos); causal softmax
+ * with scale 1/sqrt(D), GQA head map q head h -> kv head h / (Hq/Hkv).
+ * out: bf16 [Hq][D].  Split-KV over 256-row splits, merged by log-sum-exp.
+ * Workspace and errors as kvb_decode_step. */
+kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const uint16_t* k_layer,
+                                const uint16_t* v_layer, int64_t n_rows, const int32_t* pos, int64_t max_pos,
+                                uint16_t* out, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, then read and clear the device status word that kernels using
  * workspace `ws` write when a bounded wait runs out.  *code_out receives KVB_OK or
  * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */

@@ -232,3 +232,18 @@ def deviation_histogram(dev, edges) -> np.ndarray:
     for d in dev:
         counts[sum(1 for e in edges if d >= e)] += 1
     return counts
+
+
+def decode_step(s: Shape, layers: Sequence[dict], embed, final_norm, lm_head, k_cache: np.ndarray,
+                v_cache: np.ndarray, token: int, pos: int) -> tuple:
+    """One step of greedy decoding (Sec. 4): the token at position `pos` runs through
+    every layer as a single row (its K/V written into cache row `pos` of each layer,
+    attention over rows [0, pos]), then the final RMSNorm, the logits and their argmax.
+    k_cache, v_cache: [L, n_rows, Hkv, D] float64, updated in place.
+    Returns (next token, final hidden [H], logits [vocab])."""
+    x = embed_rows(embed, np.array([token]))
+    for l, lw in enumerate(layers):
+        x = layer_rows(s, lw, x, [pos], [pos], k_cache[l], v_cache[l])
+    h = rmsnorm(x, final_norm, s.rms_eps)
+    tok, logits = first_token(h, lm_head)
+    return int(tok[0]), h[0], logits[0]

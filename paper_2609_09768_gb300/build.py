@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libkvblend.so")
-SOURCES = ["api.cu", "elementwise.cu", "hkvd.cu", "gemm.cu", "attn.cu", "noalloc.cu", "lmhead.cu", "select.cu"]
+SOURCES = ["api.cu", "elementwise.cu", "hkvd.cu", "gemm.cu", "attn.cu", "noalloc.cu", "lmhead.cu", "select.cu", "decode.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

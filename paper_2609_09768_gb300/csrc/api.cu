@@ -866,6 +866,123 @@ kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, co
                          static_cast<cudaStream_t>(stream));
 }
 
+// ------------------------------------------------------------------ greedy decode
+
+struct DecodeWs {
+    int* status;
+    float *x, *qkv, *hidden, *pm, *pl, *po;
+    uint16_t *a, *attn, *h, *q;
+    unsigned long long* keys;
+    int32_t* tok;
+};
+
+static size_t decode_layout(const kvb_config* c, int64_t max_pos, void* base, DecodeWs* w) {
+    size_t off = 0;
+    char* b = static_cast<char*>(base);
+    auto take = [&](size_t bytes) -> void* {
+        void* p = b ? b + off : nullptr;
+        off = align_up(off + bytes, 256);
+        return p;
+    };
+    const int64_t H = c->hidden, F = c->mlp_dim, D = c->head_dim, Hq = c->n_q_heads, Hkv = c->n_kv_heads;
+    const int64_t S = decode_splits(max_pos);
+    w->status = static_cast<int*>(take(256));
+    w->x = static_cast<float*>(take(H * 4));
+    w->hidden = static_cast<float*>(take(H * 4));
+    w->qkv = static_cast<float*>(take((Hq + 2 * Hkv) * D * 4));
+    w->a = static_cast<uint16_t*>(take(H * 2));
+    w->q = static_cast<uint16_t*>(take(Hq * D * 2));
+    w->attn = static_cast<uint16_t*>(take(Hq * D * 2));
+    w->h = static_cast<uint16_t*>(take(F * 2));
+    w->keys = static_cast<unsigned long long*>(take(8));
+    w->tok = static_cast<int32_t*>(take(4));
+    w->pm = static_cast<float*>(take(S * Hq * 4));
+    w->pl = static_cast<float*>(take(S * Hq * 4));
+    w->po = static_cast<float*>(take(S * Hq * D * 4));
+    return off;
+}
+
+static kvb_status check_decode(const kvb_config* cfg, int64_t max_pos) {
+    KVB_TRY(check_cfg(cfg));
+    if (max_pos < 1 || max_pos > 0x7FFFFFFE) return fail(KVB_ERR_INVALID_ARG, "decode: max_pos out of range");
+    const int64_t qd = (int64_t)cfg->n_q_heads * cfg->head_dim;
+    if (cfg->hidden > KVB_DECODE_MAX_K || cfg->mlp_dim > KVB_DECODE_MAX_K || qd > KVB_DECODE_MAX_K)
+        return fail(KVB_ERR_UNSUPPORTED, "decode: hidden, mlp_dim and Hq*D must be at most %d", KVB_DECODE_MAX_K);
+    return KVB_OK;
+}
+
+kvb_status kvb_decode_workspace_size(const kvb_config* cfg, int64_t max_pos, size_t* bytes) {
+    g_err[0] = 0;
+    KVB_TRY(check_decode(cfg, max_pos));
+    if (!bytes) return fail(KVB_ERR_INVALID_ARG, "decode workspace size: bytes is NULL");
+    DecodeWs w;
+    *bytes = decode_layout(cfg, max_pos, nullptr, &w);
+    return KVB_OK;
+}
+
+kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const uint16_t* k_layer,
+                                const uint16_t* v_layer, int64_t n_rows, const int32_t* pos, int64_t max_pos,
+                                uint16_t* out, void* ws, size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    KVB_TRY(check_decode(cfg, max_pos));
+    if (n_rows < max_pos) return fail(KVB_ERR_INVALID_ARG, "decode attention: n_rows %lld < max_pos %lld",
+                                      (long long)n_rows, (long long)max_pos);
+    KVB_TRY(check_ptr(q, "q"));
+    KVB_TRY(check_ptr(k_layer, "k_layer"));
+    KVB_TRY(check_ptr(v_layer, "v_layer"));
+    KVB_TRY(check_ptr(pos, "pos"));
+    KVB_TRY(check_ptr(out, "out"));
+    DecodeWs w;
+    const size_t need = decode_layout(cfg, max_pos, nullptr, &w);
+    if (!ws || ws_bytes < need) return fail(KVB_ERR_WORKSPACE, "decode attention: workspace %zu < %zu", ws_bytes, need);
+    decode_layout(cfg, max_pos, ws, &w);
+    const float sl2 = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
+    return launch_decode_attn(q, k_layer, v_layer, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, pos, max_pos, sl2,
+                              w.pm, w.pl, w.po, out, w.status, static_cast<cudaStream_t>(stream));
+}
+
+kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
+                           const kvb_kv_cache* cache, const uint16_t* lm_head, int32_t* tokens, int32_t* pos,
+                           int64_t max_pos, float* hidden_out, void* ws, size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    KVB_TRY(check_decode(cfg, max_pos));
+    if (cfg->vocab < 1 || cfg->hidden > 8192) return fail(KVB_ERR_UNSUPPORTED, "decode: vocab >= 1, hidden <= 8192");
+    KVB_TRY(check_model(cfg, model));
+    KVB_TRY(check_rope(rope, max_pos));
+    KVB_TRY(check_cache(cfg, cache, max_pos));
+    KVB_TRY(check_ptr(lm_head, "lm_head"));
+    KVB_TRY(check_ptr(tokens, "tokens"));
+    KVB_TRY(check_ptr(pos, "pos"));
+    if (hidden_out) KVB_TRY(check_ptr(hidden_out, "hidden_out"));
+    DecodeWs w;
+    const size_t need = decode_layout(cfg, max_pos, nullptr, &w);
+    if (!ws || ws_bytes < need) return fail(KVB_ERR_WORKSPACE, "decode: workspace %zu < %zu", ws_bytes, need);
+    decode_layout(cfg, max_pos, ws, &w);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int H = cfg->hidden, F = cfg->mlp_dim, D = cfg->head_dim, Hq = cfg->n_q_heads, Hkv = cfg->n_kv_heads;
+    const int QD = Hq * D, KVD = Hkv * D;
+    const float eps = cfg->rms_eps;
+    const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));
+    float* hidden = hidden_out ? hidden_out : w.hidden;
+    KVB_TRY(launch_decode_embed(model->embed, tokens, pos, max_pos, cfg->vocab, H, w.x, w.status, st));
+    for (int l = 0; l < cfg->n_layers; ++l) {
+        const kvb_layer_weights& lw = model->layers[l];
+        uint16_t* kc = cache->k + (int64_t)l * cache->n_rows * KVD;
+        uint16_t* vc = cache->v + (int64_t)l * cache->n_rows * KVD;
+        KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, lw.attn_norm, eps, w.a, nullptr, st));
+        KVB_TRY(launch_gemv(GEMV_F32, lw.w_qkv, nullptr, QD + 2 * KVD, H, w.a, w.qkv, nullptr, st));
+        KVB_TRY(launch_qkv_finish(w.qkv, pos, max_pos, rope->cos, rope->sin, D, Hq, Hkv, w.q, kc, vc, w.status, st));
+        KVB_TRY(launch_decode_attn(w.q, kc, vc, Hq, Hkv, D, pos, max_pos, sl2, w.pm, w.pl, w.po, w.attn, w.status, st));
+        KVB_TRY(launch_gemv(GEMV_RESID, lw.w_o, nullptr, H, QD, w.attn, w.x, nullptr, st));
+        KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, lw.mlp_norm, eps, w.a, nullptr, st));
+        KVB_TRY(launch_gemv(GEMV_SWIGLU, lw.w_gate, lw.w_up, F, H, w.a, nullptr, w.h, st));
+        KVB_TRY(launch_gemv(GEMV_RESID, lw.w_down, nullptr, H, F, w.h, w.x, nullptr, st));
+    }
+    KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, model->final_norm, eps, nullptr, hidden, st));
+    KVB_TRY(launch_lmhead(lm_head, cfg->vocab, H, hidden, 1, nullptr, w.keys, w.tok, st));
+    return launch_decode_finish(w.tok, tokens, pos, max_pos, w.status, st);
+}
+
 kvb_status kvb_debug_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
     g_err[0] = 0;
     if (!ws || ws_bytes < 256 || limit_ns < 1000 || limit_ns > 4000000000ll)

@@ -103,6 +103,23 @@ kvb_status launch_window_select(const int32_t* win_start, int32_t n_win, int32_t
 kvb_status launch_deviation_histogram(const uint16_t* ka, int64_t lda, const uint16_t* kb, int64_t ldb, int64_t n,
                                       int kv_dim, const float* edges, int n_edges, float* dev,
                                       unsigned long long* hist, cudaStream_t st);
+// ---------------------------------------------------------------- greedy decode
+constexpr int KVB_DECODE_KEYS_PER_SPLIT = 256;   // cache rows per warp split of the decode attention
+constexpr int KVB_DECODE_MAX_K = 16384;          // longest input row of a decode GEMV (shared memory)
+enum GemvMode { GEMV_F32 = 0, GEMV_RESID = 1, GEMV_SWIGLU = 2 };
+int decode_splits(int64_t max_pos);
+kvb_status launch_decode_embed(const uint16_t* embed, const int32_t* tokens, const int32_t* pos, int64_t max_pos,
+                               int64_t vocab, int H, float* x, int* status, cudaStream_t st);
+kvb_status launch_gemv(int mode, const uint16_t* W, const uint16_t* W2, int64_t N, int K, const uint16_t* a,
+                       float* y_f32, uint16_t* y_bf16, cudaStream_t st);
+kvb_status launch_qkv_finish(const float* qkv, const int32_t* pos, int64_t max_pos, const float* cos_t,
+                             const float* sin_t, int D, int Hq, int Hkv, uint16_t* q_out, uint16_t* k_layer,
+                             uint16_t* v_layer, int* status, cudaStream_t st);
+kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hq, int Hkv, int D,
+                              const int32_t* pos, int64_t max_pos, float sl2, float* pm, float* pl, float* po,
+                              uint16_t* out, int* status, cudaStream_t st);
+kvb_status launch_decode_finish(const int32_t* tok, int32_t* tokens, int32_t* pos, int64_t max_pos, int* status,
+                                cudaStream_t st);
 kvb_status launch_lmhead(const uint16_t* W, int64_t vocab, int H, const float* x, int n, float* logits,
                          unsigned long long* keys, int32_t* tokens, cudaStream_t st);
 

@@ -97,6 +97,10 @@ _SIGS = {
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
     "kvb_debug_wait_timeout": (c_i32, [c_vp, c_sz, c_i64, c_vp]),
     "kvb_lm_head_argmax": (c_i32, [P(Config), c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_sz, c_vp]),
+    "kvb_decode_workspace_size": (c_i32, [P(Config), c_i64, P(c_sz)]),
+    "kvb_decode_step": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), P(KVCache), c_vp, c_vp, c_vp, c_i64,
+                                c_vp, c_vp, c_sz, c_vp]),
+    "kvb_decode_attention": (c_i32, [P(Config), c_vp, c_vp, c_vp, c_i64, c_vp, c_i64, c_vp, c_vp, c_sz, c_vp]),
     "kvb_window_select_workspace_size": (c_sz, [c_i64]),
     "kvb_window_select": (c_i32, [c_vp, c_i32, c_i32, c_i64, c_vp, c_vp, c_vp, c_sz, c_vp]),
     "kvb_key_deviation_histogram": (c_i32, [c_vp, c_i64, c_vp, c_i64, c_i64, c_i32, c_vp, c_i32, c_vp, c_vp, c_vp,
@@ -436,3 +440,42 @@ def full_prefill(cfg: Config, model: Model, rope: RopeTable, cache_k, cache_v, t
           _ptr(kv_lo, torch.int32, "kv_lo"), _ptr(final_hidden, torch.float32, "final_hidden") if n_out else None,
           n_out, C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream())
     return final_hidden, (t.as_dict() if timings else None)
+
+
+# ---------------------------------------------------------------------------------- decode
+
+def decode_workspace(cfg: Config, max_pos: int, device="cuda") -> torch.Tensor:
+    """A zeroed workspace for kvb_decode_step / kvb_decode_attention up to max_pos."""
+    n = c_sz(0)
+    _call("kvb_decode_workspace_size", C.byref(cfg), max_pos, C.byref(n))
+    return torch.zeros(n.value, dtype=torch.uint8, device=device)
+
+
+def decode_step(cfg: Config, model: Model, rope: RopeTable, cache_k, cache_v, lm_head: torch.Tensor,
+                tokens: torch.Tensor, pos: torch.Tensor, max_pos: int, hidden: Optional[torch.Tensor] = None,
+                ws: Optional[torch.Tensor] = None):
+    """One greedy decode step on the device: reads tokens[pos], writes tokens[pos + 1] and
+    the new K/V at cache row pos, increments pos (int32 [1] on the device)."""
+    if ws is None:
+        ws = decode_workspace(cfg, max_pos, tokens.device)
+    if tokens.numel() < max_pos + 1:
+        raise ValueError("tokens needs room for max_pos + 1 ids")
+    cache = kv_cache_struct(cache_k, cache_v)
+    _call("kvb_decode_step", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct), C.byref(cache),
+          _ptr(lm_head, torch.bfloat16, "lm_head"), _ptr(tokens, torch.int32, "tokens"), _ptr(pos, torch.int32, "pos"),
+          max_pos, _ptr(hidden, torch.float32, "hidden"), _ptr(ws), ws.numel(), _stream())
+    return ws
+
+
+def decode_attention(cfg: Config, q: torch.Tensor, k_layer: torch.Tensor, v_layer: torch.Tensor, pos: torch.Tensor,
+                     max_pos: int, out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None):
+    """Attention of one new row (q bf16 [Hq][D]) over cache rows [0, pos] of one layer
+    (k bf16 / v fp16, [n_rows][Hkv][D]).  Returns bf16 [Hq][D]."""
+    if out is None:
+        out = torch.empty(cfg.n_q_heads, cfg.head_dim, dtype=torch.bfloat16, device=q.device)
+    if ws is None:
+        ws = decode_workspace(cfg, max_pos, q.device)
+    _call("kvb_decode_attention", C.byref(cfg), _ptr(q, torch.bfloat16, "q"), _ptr(k_layer, torch.bfloat16, "k"),
+          _ptr(v_layer, torch.float16, "v"), k_layer.shape[0], _ptr(pos, torch.int32, "pos"), max_pos,
+          _ptr(out, torch.bfloat16, "out"), _ptr(ws), ws.numel(), _stream())
+    return out

@@ -527,3 +527,30 @@ def test_selective_prefill_with_separators_recompute_all_equals_full():
     assert np.all(sp["k"][1:, [5, 6, 12, 13]] != 0)           # recomputed in the selective layers
     kv = blend.selective_prefill(s, layers, x0, starts, 4, 0.0, cc["k"], cc["v"], forced_sel=[7])
     assert np.all(kv["k"][1:, [5, 6, 12, 13]] == 0) and np.all(kv["v"][1:, [5, 6, 12, 13]] == 0)
+
+
+def test_decode_steps_equal_a_longer_full_prefill():
+    """Two greedy decode steps after a full prefill of n tokens give the final hidden
+    states of a full prefill of n + 2 tokens at its last two rows (the appended K/V rows,
+    positions and causal range must all be right)."""
+    s = Shape(hidden=16, n_q_heads=4, n_kv_heads=2, head_dim=8, mlp_dim=24, rms_eps=1e-5, rope_theta=1e4)
+    rng = np.random.default_rng(21)
+    layers = [{"attn_norm": np.ones(16), "mlp_norm": np.ones(16),
+               "w_qkv": rng.standard_normal((64, 16)) * 0.3, "w_o": rng.standard_normal((16, 32)) * 0.3,
+               "w_gate": rng.standard_normal((24, 16)) * 0.3, "w_up": rng.standard_normal((24, 16)) * 0.3,
+               "w_down": rng.standard_normal((16, 24)) * 0.3} for _ in range(2)]
+    embed = rng.standard_normal((40, 16))
+    lm = rng.standard_normal((40, 16)) * 0.3
+    fn = np.ones(16)
+    toks = rng.integers(0, 40, 9)
+    n = 7
+    pre = blend.full_prefill(s, layers, blend.embed_rows(embed, toks[:n]))
+    kc = np.zeros((2, 9, 2, 8)); vc = np.zeros_like(kc)
+    kc[:, :n] = pre["k"]; vc[:, :n] = pre["v"]
+    t1, h1, _ = blend.decode_step(s, layers, embed, fn, lm, kc, vc, int(toks[n]), n)
+    t2, h2, l2 = blend.decode_step(s, layers, embed, fn, lm, kc, vc, int(toks[n + 1]), n + 1)
+    full = blend.full_prefill(s, layers, blend.embed_rows(embed, toks))
+    fh = llama.rmsnorm(full["x"], fn, s.rms_eps)
+    assert np.allclose(h1, fh[n], rtol=1e-10, atol=1e-12) and np.allclose(h2, fh[n + 1], rtol=1e-10, atol=1e-12)
+    assert np.allclose(kc, full["k"], rtol=1e-10, atol=1e-12)
+    assert t2 == int(np.argmax(fh[n + 1] @ lm.T)) and t1 == int(np.argmax(fh[n] @ lm.T))
