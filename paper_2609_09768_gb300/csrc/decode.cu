@@ -11,12 +11,13 @@
 //   qkv_finish        - RoPE at `pos` on q and k (fp32, then bf16), K and V written
 //                       into cache row `pos` (V as bf16-rounded fp16, like the prefill)
 //   decode_attn       - split-KV attention of the new row over cache rows [0, pos]:
-//                       one warp per split of DEC_KEYS keys and kv head, lanes over head
+//                       one warp per split of 128 keys and kv head, lanes over head
 //                       dims; the G q heads sharing the kv head and 32/G keys give 32
 //                       partial dot products per step, summed with one 31-shuffle
-//                       reduce-scatter; online softmax per head in fp32; partial
-//                       (max, sum, O) per split
-//   decode_combine    - log-sum-exp merge of the splits -> bf16 attention output
+//                       reduce-scatter; online softmax per head in fp32; the next
+//                       step's K/V loads are issued before this step's arithmetic; the 8
+//                       warps of a CTA merge their (max, sum, O) in shared memory
+//   decode_combine    - log-sum-exp merge of the CTA partials -> bf16 attention output
 //   decode_finish     - tokens[pos + 1] = argmax, pos += 1
 // The position and the token live in device memory, so a step needs no host value that
 // changes from one step to the next.  Kernels that read `pos` check 0 <= pos < max_pos
@@ -139,24 +140,44 @@ __global__ void qkv_finish_kernel(const float* __restrict__ qkv, const int32_t* 
     }
 }
 
-// One warp = one split of `keys_per_split` cache rows for kv head blockIdx.y.
+// Unpack one lane's DPL head dims of a key (bf16) or value (fp16) row from raw words.
+template <int DPL>
+struct RowBits {
+    uint32_t w[DPL / 2];
+};
+template <int DPL>
+KVB_DEV RowBits<DPL> load_row(const uint16_t* p) {
+    RowBits<DPL> r;
+    if constexpr (DPL == 4) {
+        const uint2 u = __ldcs(reinterpret_cast<const uint2*>(p));
+        r.w[0] = u.x; r.w[1] = u.y;
+    } else {
+        r.w[0] = __ldcs(reinterpret_cast<const unsigned int*>(p));
+    }
+    return r;
+}
+
+// One CTA = eight consecutive splits of KVB_DECODE_KEYS_PER_SPLIT cache rows for kv head
+// blockIdx.y, one warp per split; the warps' partial results are merged in shared memory
+// and the CTA writes one partial (max, sum, O) per q head.
 template <int D, int G>
-__global__ void __launch_bounds__(ATT_THREADS)
+__global__ void __launch_bounds__(ATT_THREADS, 2)
 decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ kc, const uint16_t* __restrict__ vc,
-                   int Hkv, const int32_t* __restrict__ pos_ptr, int64_t max_pos, int keys_per_split, int n_splits,
-                   float scale_log2, float* __restrict__ pm, float* __restrict__ pl, float* __restrict__ po,
-                   int* status) {
+                   int Hkv, const int32_t* __restrict__ pos_ptr, int64_t max_pos, int n_blocks, float scale_log2,
+                   float* __restrict__ pm, float* __restrict__ pl, float* __restrict__ po, int* status) {
     constexpr int DPL = D / 32;      // head dims per lane
     constexpr int KS = 32 / G;       // keys per step: KS * G = 32 partial dot products
+    constexpr int WARPS = ATT_THREADS / 32;
+    __shared__ float sm_m[WARPS][G], sm_l[WARPS][G];
+    __shared__ float sm_o[WARPS][G][D];
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
-    const int lane = threadIdx.x & 31;
-    const int split = blockIdx.x * (ATT_THREADS / 32) + (threadIdx.x >> 5);
-    if (split >= n_splits) return;
+    if ((int)blockIdx.x >= n_blocks) return;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = blockIdx.y;
     const int Hq = Hkv * G;
-    const int64_t start = (int64_t)split * keys_per_split;
-    int64_t end = start + keys_per_split;
+    const int64_t start = ((int64_t)blockIdx.x * WARPS + warp) * KVB_DECODE_KEYS_PER_SPLIT;
+    int64_t end = start + KVB_DECODE_KEYS_PER_SPLIT;
     if (end > (int64_t)pos + 1) end = (int64_t)pos + 1;
 
     float qv[G][DPL];
@@ -164,7 +185,6 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
     for (int h = 0; h < G; ++h)
 #pragma unroll
         for (int e = 0; e < DPL; ++e) qv[h][e] = bf16_to_f(q[(g * G + h) * D + lane * DPL + e]);
-
     float o[G][DPL];
 #pragma unroll
     for (int h = 0; h < G; ++h)
@@ -175,42 +195,37 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
     const int64_t row_stride = (int64_t)Hkv * D;
     const uint16_t* kbase = kc + (int64_t)g * D + lane * DPL;
     const uint16_t* vbase = vc + (int64_t)g * D + lane * DPL;
-    for (int64_t k0 = start; k0 < end; k0 += KS) {
-        float kf[KS][DPL], vf[KS][DPL];
+    RowBits<DPL> ck[KS], cv[KS], nk[KS], nv[KS];
+    auto fetch = [&](int64_t k0, RowBits<DPL>* kr, RowBits<DPL>* vr) {
 #pragma unroll
         for (int k = 0; k < KS; ++k) {
-            const int64_t key = k0 + k;
-            if (key < end) {
-                if constexpr (DPL == 4) {
-                    const uint2 kw = __ldcs(reinterpret_cast<const uint2*>(kbase + key * row_stride));
-                    const uint2 vw = __ldcs(reinterpret_cast<const uint2*>(vbase + key * row_stride));
-                    kf[k][0] = bf16_lo(kw.x); kf[k][1] = bf16_hi(kw.x); kf[k][2] = bf16_lo(kw.y); kf[k][3] = bf16_hi(kw.y);
-                    const float2 va = __half22float2(*reinterpret_cast<const __half2*>(&vw.x));
-                    const float2 vb = __half22float2(*reinterpret_cast<const __half2*>(&vw.y));
-                    vf[k][0] = va.x; vf[k][1] = va.y; vf[k][2] = vb.x; vf[k][3] = vb.y;
-                } else {
-                    const uint32_t kw = __ldcs(reinterpret_cast<const unsigned int*>(kbase + key * row_stride));
-                    const uint32_t vw = __ldcs(reinterpret_cast<const unsigned int*>(vbase + key * row_stride));
-                    kf[k][0] = bf16_lo(kw); kf[k][1] = bf16_hi(kw);
-                    const float2 va = __half22float2(*reinterpret_cast<const __half2*>(&vw));
-                    vf[k][0] = va.x; vf[k][1] = va.y;
-                }
+            if (k0 + k < end) {
+                kr[k] = load_row<DPL>(kbase + (k0 + k) * row_stride);
+                vr[k] = load_row<DPL>(vbase + (k0 + k) * row_stride);
             } else {
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) { kf[k][e] = 0.f; vf[k][e] = 0.f; }
+                for (int i = 0; i < DPL / 2; ++i) { kr[k].w[i] = 0u; vr[k].w[i] = 0u; }
             }
         }
-        // partial dot products of this lane's head dims: index k * G + h
+    };
+    if (start < end) fetch(start, ck, cv);
+    for (int64_t k0 = start; k0 < end; k0 += KS) {
+        // loads of the next step go out before this step's arithmetic
+        if (k0 + KS < end) fetch(k0 + KS, nk, nv);
         float sc[32];
 #pragma unroll
-        for (int k = 0; k < KS; ++k)
+        for (int k = 0; k < KS; ++k) {
+            float kf[DPL];
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
 #pragma unroll
             for (int h = 0; h < G; ++h) {
                 float acc = 0.f;
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[k][e], acc);
+                for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[e], acc);
                 sc[k * G + h] = acc;
             }
+        }
         // reduce-scatter: afterwards lane L holds the full dot product of index L
 #pragma unroll
         for (int off = 16; off >= 1; off >>= 1) {
@@ -222,9 +237,8 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
                 sc[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
             }
         }
-        const int my_key = lane / G;
         float t = sc[0] * scale_log2;
-        if (k0 + my_key >= end) t = -INFINITY;
+        if (k0 + lane / G >= end) t = -INFINITY;
         // online softmax of head lane % G over this step's keys
         float mx = t;
 #pragma unroll
@@ -242,43 +256,89 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
             const float ah = __shfl_sync(0xffffffffu, alpha, h);
 #pragma unroll
             for (int e = 0; e < DPL; ++e) o[h][e] *= ah;
+        }
 #pragma unroll
-            for (int k = 0; k < KS; ++k) {
+        for (int k = 0; k < KS; ++k) {
+            float vf[DPL];
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&cv[k].w[i]));
+                vf[2 * i] = f.x; vf[2 * i + 1] = f.y;
+            }
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
                 const float pk = __shfl_sync(0xffffffffu, pv, k * G + h);
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk, vf[k][e], o[h][e]);
+                for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk, vf[e], o[h][e]);
             }
         }
+#pragma unroll
+        for (int k = 0; k < KS; ++k) { ck[k] = nk[k]; cv[k] = nv[k]; }
     }
-    const int64_t base = (int64_t)split * Hq + g * G;
+    // merge the warps of this CTA
 #pragma unroll
     for (int h = 0; h < G; ++h)
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) po[(base + h) * D + lane * DPL + e] = o[h][e];
-    if (lane < G) {
-        pm[base + lane] = m_run;
-        pl[base + lane] = l_run;
+        for (int e = 0; e < DPL; ++e) sm_o[warp][h][lane * DPL + e] = o[h][e];
+    if (lane < G) { sm_m[warp][lane] = m_run; sm_l[warp][lane] = l_run; }
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * Hq + g * G;
+    for (int i = threadIdx.x; i < G * D; i += ATT_THREADS) {
+        const int h = i / D, d = i % D;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < WARPS; ++w) M = fmaxf(M, sm_m[w][h]);
+        float L = 0.f, O = 0.f;
+#pragma unroll
+        for (int w = 0; w < WARPS; ++w) {
+            const float c = (sm_m[w][h] == -INFINITY) ? 0.f : exp2f(sm_m[w][h] - M);
+            L += c * sm_l[w][h];
+            O += c * sm_o[w][h][d];
+        }
+        po[(base + h) * D + d] = O;
+        if (d == 0) { pm[base + h] = M; pl[base + h] = L; }
     }
 }
 
-// One block per q head, one thread per head dim.
+// One block per q head: COMB_GROUPS groups of D threads, each over every COMB_GROUPS-th CTA
+// partial, then merged in shared memory.
+constexpr int COMB_GROUPS = 4;
 __global__ void decode_combine_kernel(const float* __restrict__ pm, const float* __restrict__ pl,
                                       const float* __restrict__ po, const int32_t* __restrict__ pos_ptr,
-                                      int64_t max_pos, int keys_per_split, int Hq, int D, uint16_t* __restrict__ out,
+                                      int64_t max_pos, int keys_per_block, int Hq, int D, uint16_t* __restrict__ out,
                                       int* status) {
+    __shared__ float s_m[COMB_GROUPS], s_l[COMB_GROUPS];
+    __shared__ float s_o[COMB_GROUPS][128];
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
-    const int hq = blockIdx.x, d = threadIdx.x;
-    const int n = (pos + keys_per_split) / keys_per_split;   // splits holding keys [0, pos]
+    const int hq = blockIdx.x, d = threadIdx.x % D, grp = threadIdx.x / D;
+    const int n = (pos + keys_per_block) / keys_per_block;   // CTA partials holding keys [0, pos]
     float M = -INFINITY;
-    for (int s = 0; s < n; ++s) M = fmaxf(M, pm[(int64_t)s * Hq + hq]);
+    for (int s = grp; s < n; s += COMB_GROUPS) M = fmaxf(M, pm[(int64_t)s * Hq + hq]);
     float L = 0.f, O = 0.f;
-    for (int s = 0; s < n; ++s) {
-        const float w = exp2f(pm[(int64_t)s * Hq + hq] - M);
+#pragma unroll 4
+    for (int s = grp; s < n; s += COMB_GROUPS) {
+        const float ms = pm[(int64_t)s * Hq + hq];
+        const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
         L += w * pl[(int64_t)s * Hq + hq];
         O += w * po[((int64_t)s * Hq + hq) * D + d];
     }
-    if (d < D) out[hq * D + d] = __bfloat16_as_ushort(__float2bfloat16_rn(L > 0.f ? O / L : 0.f));
+    if (d == 0) { s_m[grp] = M; s_l[grp] = L; }
+    s_o[grp][d] = O;
+    __syncthreads();
+    if (grp == 0) {
+        float MM = -INFINITY;
+#pragma unroll
+        for (int q2 = 0; q2 < COMB_GROUPS; ++q2) MM = fmaxf(MM, s_m[q2]);
+        float LL = 0.f, OO = 0.f;
+#pragma unroll
+        for (int q2 = 0; q2 < COMB_GROUPS; ++q2) {
+            const float w = (s_m[q2] == -INFINITY) ? 0.f : exp2f(s_m[q2] - MM);
+            LL += w * s_l[q2];
+            OO += w * s_o[q2][d];
+        }
+        out[hq * D + d] = __bfloat16_as_ushort(__float2bfloat16_rn(LL > 0.f ? OO / LL : 0.f));
+    }
 }
 
 __global__ void decode_finish_kernel(const int32_t* __restrict__ tok, int32_t* __restrict__ tokens,
@@ -291,11 +351,11 @@ __global__ void decode_finish_kernel(const int32_t* __restrict__ tok, int32_t* _
 
 template <int D, int G>
 kvb_status run_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hkv, const int32_t* pos,
-                    int64_t max_pos, int n_splits, float sl2, float* pm, float* pl, float* po, int* status,
+                    int64_t max_pos, int n_blocks, float sl2, float* pm, float* pl, float* po, int* status,
                     cudaStream_t st) {
-    const dim3 grid((unsigned)((n_splits + ATT_THREADS / 32 - 1) / (ATT_THREADS / 32)), (unsigned)Hkv);
-    decode_attn_kernel<D, G><<<grid, ATT_THREADS, 0, st>>>(q, kc, vc, Hkv, pos, max_pos, KVB_DECODE_KEYS_PER_SPLIT,
-                                                           n_splits, sl2, pm, pl, po, status);
+    const dim3 grid((unsigned)n_blocks, (unsigned)Hkv);
+    decode_attn_kernel<D, G><<<grid, ATT_THREADS, 0, st>>>(q, kc, vc, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po,
+                                                           status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode attention launch");
 }
@@ -353,8 +413,10 @@ kvb_status launch_qkv_finish(const float* qkv, const int32_t* pos, int64_t max_p
     return cuda_ok(cudaGetLastError(), "qkv finish launch");
 }
 
+// CTA partials of the decode attention for positions below max_pos
 int decode_splits(int64_t max_pos) {
-    return (int)((max_pos + KVB_DECODE_KEYS_PER_SPLIT - 1) / KVB_DECODE_KEYS_PER_SPLIT);
+    const int64_t per_block = (int64_t)KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32);
+    return (int)((max_pos + per_block - 1) / per_block);
 }
 
 kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hq, int Hkv, int D,
@@ -370,8 +432,8 @@ kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint1
     else if (D == 64 && G == 4) s = run_attn<64, 4>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
     else return fail(KVB_ERR_UNSUPPORTED, "decode attention: head_dim %d with %d q heads per kv head not built", D, G);
     if (s != KVB_OK) return s;
-    decode_combine_kernel<<<(unsigned)Hq, (unsigned)D, 0, st>>>(pm, pl, po, pos, max_pos, KVB_DECODE_KEYS_PER_SPLIT,
-                                                                Hq, D, out, status);
+    decode_combine_kernel<<<(unsigned)Hq, (unsigned)(D * COMB_GROUPS), 0, st>>>(
+        pm, pl, po, pos, max_pos, KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32), Hq, D, out, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode combine launch");
 }

@@ -4,6 +4,8 @@
     python -m paper_2609_09768_gb300.profile_case dense --n-kv 16384
     python -m paper_2609_09768_gb300.profile_case gemm  --m 18713 --which qkv|o|gateup|down
     python -m paper_2609_09768_gb300.profile_case realign --n-ctx 123904 --layers 2
+    python -m paper_2609_09768_gb300.profile_case decode_attn --n-kv 124032
+    python -m paper_2609_09768_gb300.profile_case decode_step --n-kv 128 --layers 4
 
 Shapes are the Llama-3.1-8B layer (H 4096, 32 q / 8 kv heads, D 128, F 14336).  The
 selected rows of `attn` are drawn uniformly over the context (as the HKVD choice of
@@ -23,7 +25,7 @@ from . import kvblend as kvb
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attn", "dense", "gemm", "realign"])
+    ap.add_argument("kernel", choices=["attn", "dense", "gemm", "realign", "decode_attn", "decode_step"])
     ap.add_argument("--m", type=int, default=18713)
     ap.add_argument("--n-kv", type=int, default=124032)
     ap.add_argument("--n-ctx", type=int, default=123904)
@@ -75,6 +77,38 @@ def main():
             fn = lambda: kvb.mlp_rows(cfg, lws, attn, x, wsl)
             flop = 2.0 * m * H * (Hq * D + 3 * F)
         out.update(m=m, which=("o+gateup+down (mlp_rows)" if a.which != "qkv" else "qkv"))
+    elif a.kernel == "decode_attn":
+        n_kv = a.n_kv
+        q = torch.randn(Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        kc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16).to(torch.float16)
+        pos = torch.tensor([n_kv - 1], dtype=torch.int32, device=dev)
+        ws = kvb.decode_workspace(cfg, n_kv, dev)
+        o = torch.empty(Hq, D, dtype=torch.bfloat16, device=dev)
+        fn = lambda: kvb.decode_attention(cfg, q, kc, vc, pos, n_kv, out=o, ws=ws)
+        flop = None
+        out.update(bytes=float(n_kv) * Hkv * D * 2 * 2, n_kv=n_kv)
+    elif a.kernel == "decode_step":
+        # a decode step of an a.layers-layer model at position n_kv - 1 (step time minus the
+        # lm_head is per-layer GEMV + attention time)
+        shp = shape.with_layers(a.layers)
+        cfgl = kvb.config(shp)
+        model = kvb.Model(synth.make_model(shp, 0, dev))
+        lm = synth.make_lm_head(shp, 0, dev)
+        n_kv = a.n_kv
+        rope = kvb.RopeTable(cfgl, n_kv, dev)
+        kc = torch.randn(a.layers, n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn(a.layers, n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16).to(torch.float16)
+        tokens = torch.zeros(n_kv + 1, dtype=torch.int32, device=dev)
+        pos = torch.tensor([n_kv - 1], dtype=torch.int32, device=dev)
+        ws = kvb.decode_workspace(cfgl, n_kv, dev)
+
+        def fn():
+            pos.fill_(n_kv - 1)
+            kvb.decode_step(cfgl, model, rope, kc, vc, lm, tokens, pos, n_kv, ws=ws)
+        flop = None
+        wb = a.layers * 2.0 * (shp.qkv_dim * H + H * shp.q_dim + 3 * H * F) + shp.vocab * H * 2.0
+        out.update(bytes=wb + a.layers * float(n_kv) * Hkv * D * 4, layers=a.layers, n_kv=n_kv)
     else:
         L, n_ctx = a.layers, a.n_ctx
         ks = torch.randn(L, n_ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
