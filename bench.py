@@ -391,9 +391,9 @@ def run_ours(args, wl, rank: int, world: int) -> None:
             kvb.decode_step(cfg, model, rope, ck, cv, lm, tokens, pos, cap, ws=dws)
         b.record()
         torch.cuda.synchronize()
-        # embed; per layer 2 RMSNorms, 4 GEMVs, RoPE/append, attention + combine; final norm,
-        # lm_head + argmax, position/token update
-        launches = 1 + 9 * L + 1 + 2 + 1
+        # embed; per layer 4 GEMVs (RMSNorm, RoPE and the K/V append fused into them),
+        # attention + combine; final norm, lm_head + argmax, position/token update
+        launches = 1 + 6 * L + 1 + 2 + 1
         dec_ms = a.elapsed_time(b) / max(n_dec - 1, 1)
         assert kvb.device_status(dws) == 0 and int(pos.item()) == N + n_dec
         p_mid = N + n_dec // 2

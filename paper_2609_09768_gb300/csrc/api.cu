@@ -870,7 +870,7 @@ kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, co
 
 struct DecodeWs {
     int* status;
-    float *x, *qkv, *hidden, *pm, *pl, *po;
+    float *x, *hidden, *pm, *pl, *po;
     uint16_t *a, *attn, *h, *q;
     unsigned long long* keys;
     int32_t* tok;
@@ -885,11 +885,10 @@ static size_t decode_layout(const kvb_config* c, int64_t max_pos, void* base, De
         return p;
     };
     const int64_t H = c->hidden, F = c->mlp_dim, D = c->head_dim, Hq = c->n_q_heads, Hkv = c->n_kv_heads;
-    const int64_t S = decode_splits(max_pos);
+    const int64_t S = decode_splits(max_pos, (int)Hkv);   // CTA partials per q head
     w->status = static_cast<int*>(take(256));
     w->x = static_cast<float*>(take(H * 4));
     w->hidden = static_cast<float*>(take(H * 4));
-    w->qkv = static_cast<float*>(take((Hq + 2 * Hkv) * D * 4));
     w->a = static_cast<uint16_t*>(take(H * 2));
     w->q = static_cast<uint16_t*>(take(Hq * D * 2));
     w->attn = static_cast<uint16_t*>(take(Hq * D * 2));
@@ -965,18 +964,32 @@ kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const 
     const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));
     float* hidden = hidden_out ? hidden_out : w.hidden;
     KVB_TRY(launch_decode_embed(model->embed, tokens, pos, max_pos, cfg->vocab, H, w.x, w.status, st));
+    GemvArgs ga{};
+    ga.eps = eps;
+    ga.pos = pos;
+    ga.max_pos = max_pos;
+    ga.cos_t = rope->cos;
+    ga.sin_t = rope->sin;
+    ga.D = D; ga.Hq = Hq; ga.Hkv = Hkv;
+    ga.status = w.status;
     for (int l = 0; l < cfg->n_layers; ++l) {
         const kvb_layer_weights& lw = model->layers[l];
         uint16_t* kc = cache->k + (int64_t)l * cache->n_rows * KVD;
         uint16_t* vc = cache->v + (int64_t)l * cache->n_rows * KVD;
-        KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, lw.attn_norm, eps, w.a, nullptr, st));
-        KVB_TRY(launch_gemv(GEMV_F32, lw.w_qkv, nullptr, QD + 2 * KVD, H, w.a, w.qkv, nullptr, st));
-        KVB_TRY(launch_qkv_finish(w.qkv, pos, max_pos, rope->cos, rope->sin, D, Hq, Hkv, w.q, kc, vc, w.status, st));
+        GemvArgs qkv = ga;                     // RMSNorm + QKV + RoPE + K/V append
+        qkv.W = lw.w_qkv; qkv.K = H; qkv.x = w.x; qkv.g = lw.attn_norm;
+        qkv.q_out = w.q; qkv.k_layer = kc; qkv.v_layer = vc;
+        KVB_TRY(launch_gemv(GEMV_QKV, qkv, st));
         KVB_TRY(launch_decode_attn(w.q, kc, vc, Hq, Hkv, D, pos, max_pos, sl2, w.pm, w.pl, w.po, w.attn, w.status, st));
-        KVB_TRY(launch_gemv(GEMV_RESID, lw.w_o, nullptr, H, QD, w.attn, w.x, nullptr, st));
-        KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, lw.mlp_norm, eps, w.a, nullptr, st));
-        KVB_TRY(launch_gemv(GEMV_SWIGLU, lw.w_gate, lw.w_up, F, H, w.a, nullptr, w.h, st));
-        KVB_TRY(launch_gemv(GEMV_RESID, lw.w_down, nullptr, H, F, w.h, w.x, nullptr, st));
+        GemvArgs o = ga;                       // x += O-proj(attention)
+        o.W = lw.w_o; o.N = H; o.K = QD; o.a = w.attn; o.y_f32 = w.x;
+        KVB_TRY(launch_gemv(GEMV_RESID, o, st));
+        GemvArgs mlp = ga;                     // h = SwiGLU(RMSNorm(x))
+        mlp.W = lw.w_gate; mlp.W2 = lw.w_up; mlp.N = F; mlp.K = H; mlp.x = w.x; mlp.g = lw.mlp_norm; mlp.y_bf16 = w.h;
+        KVB_TRY(launch_gemv(GEMV_SWIGLU, mlp, st));
+        GemvArgs down = ga;                    // x += down(h)
+        down.W = lw.w_down; down.N = H; down.K = F; down.a = w.h; down.y_f32 = w.x;
+        KVB_TRY(launch_gemv(GEMV_RESID, down, st));
     }
     KVB_TRY(launch_rmsnorm(w.x, nullptr, 1, H, model->final_norm, eps, nullptr, hidden, st));
     KVB_TRY(launch_lmhead(lm_head, cfg->vocab, H, hidden, 1, nullptr, w.keys, w.tok, st));

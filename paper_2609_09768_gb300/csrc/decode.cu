@@ -4,12 +4,14 @@
 // for Llama-3.1-8B, and every layer's cache up to the current position), so the
 // kernels are CUDA-core kernels built for streaming, not tensor-core tiles:
 //   decode_embed      - x = embed[tokens[pos]] (fp32)
-//   gemv_kernel       - y = W a for one bf16 activation row held in shared memory;
-//                       warp per output row, eight 16-byte weight loads per lane in
-//                       flight; epilogues: fp32 out, residual add, SwiGLU (gate and up
-//                       rows in the same warp)
-//   qkv_finish        - RoPE at `pos` on q and k (fp32, then bf16), K and V written
-//                       into cache row `pos` (V as bf16-rounded fp16, like the prefill)
+//   gemv_kernel       - y = W a for one activation row held in shared memory as bf16;
+//                       warp per output row (or row pair), 16-byte weight loads, 8-16 per
+//                       lane in flight.  QKV and SwiGLU normalise the residual row
+//                       themselves (RMSNorm prologue in every block); QKV computes the two
+//                       rows of a rotation pair in one warp, applies RoPE at `pos` and writes
+//                       q and the cache's K/V row `pos` (V as bf16-rounded fp16, like the
+//                       prefill); the residual mode adds into x; SwiGLU computes gate and
+//                       up rows in one warp
 //   decode_attn       - split-KV attention of the new row over cache rows [0, pos]:
 //                       one warp per split of 128 keys and kv head, lanes over head
 //                       dims; the G q heads sharing the kv head and 32/G keys give 32
@@ -55,88 +57,141 @@ __global__ void decode_embed_kernel(const uint16_t* __restrict__ embed, const in
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < H; i += gridDim.x * blockDim.x) x[i] = bf16_to_f(row[i]);
 }
 
-template <int MODE>
-__global__ void __launch_bounds__(GEMV_THREADS)
-gemv_kernel(const uint16_t* __restrict__ W, const uint16_t* __restrict__ W2, int64_t N, int K,
-            const uint16_t* __restrict__ a, float* __restrict__ y_f32, uint16_t* __restrict__ y_bf16) {
-    extern __shared__ float av[];   // [K]
-    for (int i = threadIdx.x; i < K; i += blockDim.x) av[i] = bf16_to_f(a[i]);
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+// Dot products of one or two bf16 weight rows with the bf16 activation row in shared memory,
+// BATCH 16-byte loads per lane per row in flight; every lane returns the full sums.
+template <bool TWO, int BATCH>
+KVB_DEV void dot_rows(const uint16_t* __restrict__ w1, const uint16_t* __restrict__ w2, const uint16_t* act, int K,
+                      int lane, float& s1, float& s2) {
+    const uint4* r1 = reinterpret_cast<const uint4*>(w1);
+    const uint4* r2 = reinterpret_cast<const uint4*>(w2);
+    const uint4* av = reinterpret_cast<const uint4*>(act);
     const int vec = K / 8;
-    for (int64_t n = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); n < N; n += warps) {
-        const uint4* wr = reinterpret_cast<const uint4*>(W + n * K);
-        const uint4* wr2 = reinterpret_cast<const uint4*>((MODE == GEMV_SWIGLU ? W2 : W) + n * K);
-        float acc = 0.f, acc2 = 0.f;
-        for (int c0 = lane; c0 < vec; c0 += 32 * GEMV_BATCH) {
-            uint4 w[GEMV_BATCH], w2[GEMV_BATCH];
+    float acc = 0.f, acc2 = 0.f;
+    for (int c0 = lane; c0 < vec; c0 += 32 * BATCH) {
+        uint4 wa[BATCH], wb[TWO ? BATCH : 1];
 #pragma unroll
-            for (int u = 0; u < GEMV_BATCH; ++u) {
-                const int c = c0 + 32 * u;
-                w[u] = c < vec ? __ldcs(wr + c) : make_uint4(0u, 0u, 0u, 0u);
-                if (MODE == GEMV_SWIGLU) w2[u] = c < vec ? __ldcs(wr2 + c) : make_uint4(0u, 0u, 0u, 0u);
+        for (int u = 0; u < BATCH; ++u) {
+            const int c = c0 + 32 * u;
+            wa[u] = c < vec ? __ldcs(r1 + c) : make_uint4(0u, 0u, 0u, 0u);
+            if constexpr (TWO) wb[u] = c < vec ? __ldcs(r2 + c) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < BATCH; ++u) {
+            const int c = c0 + 32 * u;
+            if (c >= vec) break;
+            const uint4 xv = av[c];
+            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+            const uint32_t ww[4] = {wa[u].x, wa[u].y, wa[u].z, wa[u].w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                acc = fmaf(bf16_lo(ww[e]), bf16_lo(xw[e]), acc);
+                acc = fmaf(bf16_hi(ww[e]), bf16_hi(xw[e]), acc);
             }
-#pragma unroll
-            for (int u = 0; u < GEMV_BATCH; ++u) {
-                const int c = c0 + 32 * u;
-                if (c >= vec) break;
-                const float4* xr = reinterpret_cast<const float4*>(av + c * 8);
-                const float4 x0 = xr[0], x1 = xr[1];
-                const float xs[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-                const uint32_t ww[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+            if constexpr (TWO) {
+                const uint32_t vw[4] = {wb[u].x, wb[u].y, wb[u].z, wb[u].w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    acc = fmaf(bf16_lo(ww[e]), xs[2 * e], acc);
-                    acc = fmaf(bf16_hi(ww[e]), xs[2 * e + 1], acc);
-                }
-                if (MODE == GEMV_SWIGLU) {
-                    const uint32_t w2w[4] = {w2[u].x, w2[u].y, w2[u].z, w2[u].w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        acc2 = fmaf(bf16_lo(w2w[e]), xs[2 * e], acc2);
-                        acc2 = fmaf(bf16_hi(w2w[e]), xs[2 * e + 1], acc2);
-                    }
+                    acc2 = fmaf(bf16_lo(vw[e]), bf16_lo(xw[e]), acc2);
+                    acc2 = fmaf(bf16_hi(vw[e]), bf16_hi(xw[e]), acc2);
                 }
             }
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            acc += __shfl_xor_sync(0xffffffffu, acc, o);
-            if (MODE == GEMV_SWIGLU) acc2 += __shfl_xor_sync(0xffffffffu, acc2, o);
-        }
-        if (lane == 0) {
-            if (MODE == GEMV_F32) y_f32[n] = acc;
-            if (MODE == GEMV_RESID) y_f32[n] += acc;
-            if (MODE == GEMV_SWIGLU)
-                y_bf16[n] = __bfloat16_as_ushort(__float2bfloat16_rn(acc / (1.0f + __expf(-acc)) * acc2));
-        }
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if constexpr (TWO) acc2 += __shfl_xor_sync(0xffffffffu, acc2, o);
+    }
+    s1 = acc;
+    s2 = acc2;
 }
 
-// Threads: (Hq + Hkv) * D/2 rotation pairs, then Hkv * D values of V.
-__global__ void qkv_finish_kernel(const float* __restrict__ qkv, const int32_t* __restrict__ pos_ptr, int64_t max_pos,
-                                  const float* __restrict__ cos_t, const float* __restrict__ sin_t, int D, int Hq,
-                                  int Hkv, uint16_t* __restrict__ q_out, uint16_t* __restrict__ k_layer,
-                                  uint16_t* __restrict__ v_layer, int* status) {
-    int pos;
-    if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
-    const int half = D / 2;
-    const int n_rot = (Hq + Hkv) * half;
-    const int t = blockIdx.x * blockDim.x + threadIdx.x;
-    if (t < n_rot) {
-        const int h = t / half, i = t % half;
-        const float a = qkv[h * D + i], b = qkv[h * D + i + half];
-        const float c = cos_t[(int64_t)pos * half + i], s = sin_t[(int64_t)pos * half + i];
-        const float y1 = a * c - b * s;
-        const float y2 = b * c + a * s;
-        uint16_t* dst = h < Hq ? q_out + h * D : k_layer + ((int64_t)pos * Hkv + (h - Hq)) * D;
-        dst[i] = __bfloat16_as_ushort(__float2bfloat16_rn(y1));
-        dst[i + half] = __bfloat16_as_ushort(__float2bfloat16_rn(y2));
-    } else if (t < n_rot + Hkv * D) {
-        const int j = t - n_rot;
-        const float v = __bfloat162float(__float2bfloat16_rn(qkv[(Hq + Hkv) * D + j]));
-        v_layer[(int64_t)pos * Hkv * D + j] = __half_as_ushort(__float2half_rn(v));
+// One GEMV of a decode step.  The activation row is put in shared memory as bf16:
+//   GEMV_QKV, GEMV_SWIGLU: RMSNorm(x) * gain of the fp32 residual row x (each block
+//                          normalises it itself: no separate norm launch);
+//   GEMV_RESID:            the bf16 row `a` as given.
+// Work units per warp:
+//   GEMV_QKV    - a rotation pair (rows i and i + D/2 of a q or k head): RoPE at `pos`,
+//                 bf16 q or cache K row `pos`; or one V row: cache V row `pos`
+//   GEMV_RESID  - one row: x[n] += y
+//   GEMV_SWIGLU - gate row n and up row n: h[n] = bf16(silu(gate) * up)
+template <int MODE>
+__global__ void __launch_bounds__(GEMV_THREADS)
+gemv_kernel(const GemvArgs p) {
+    extern __shared__ __align__(16) uint16_t act[];   // [K]
+    __shared__ float red[GEMV_THREADS / 32];
+    const int K = p.K;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int pos = 0;
+    if constexpr (MODE == GEMV_QKV) {
+        if (!pos_ok(p.pos, p.max_pos, p.status, pos)) return;
+    }
+    if constexpr (MODE == GEMV_RESID) {
+        for (int i = threadIdx.x; i < K / 8; i += blockDim.x)
+            reinterpret_cast<uint4*>(act)[i] = reinterpret_cast<const uint4*>(p.a)[i];
+    } else {
+        const float4* x4 = reinterpret_cast<const float4*>(p.x);
+        float ss = 0.f;
+        for (int i = threadIdx.x; i < K / 4; i += blockDim.x) {
+            const float4 v = x4[i];
+            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        if (lane == 0) red[warp] = ss;
+        __syncthreads();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < GEMV_THREADS / 32; ++w) tot += red[w];
+        const float inv = rsqrtf(tot / (float)K + p.eps);
+        const float4* g4 = reinterpret_cast<const float4*>(p.g);
+        for (int i = threadIdx.x; i < K / 4; i += blockDim.x) {
+            const float4 v = x4[i], gg = __ldg(g4 + i);
+            reinterpret_cast<uint2*>(act)[i] =
+                make_uint2(pack_bf16(v.x * inv * gg.x, v.y * inv * gg.y), pack_bf16(v.z * inv * gg.z, v.w * inv * gg.w));
+        }
+    }
+    __syncthreads();
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+    const int64_t first = (int64_t)blockIdx.x * (blockDim.x / 32) + warp;
+    if constexpr (MODE == GEMV_QKV) {
+        const int D = p.D, half = D / 2, Hq = p.Hq, Hkv = p.Hkv;
+        const int64_t n_pairs = (int64_t)(Hq + Hkv) * half, n_units = n_pairs + (int64_t)Hkv * D;
+        for (int64_t u = first; u < n_units; u += warps) {
+            if (u < n_pairs) {
+                const int h = (int)(u / half), i = (int)(u % half);
+                float a, b;
+                dot_rows<true, 8>(p.W + ((int64_t)h * D + i) * K, p.W + ((int64_t)h * D + i + half) * K, act, K, lane,
+                                  a, b);
+                if (lane == 0) {
+                    const float c = p.cos_t[(int64_t)pos * half + i], sn = p.sin_t[(int64_t)pos * half + i];
+                    const float y1 = a * c - b * sn;
+                    const float y2 = b * c + a * sn;
+                    uint16_t* dst = h < Hq ? p.q_out + h * D : p.k_layer + ((int64_t)pos * Hkv + (h - Hq)) * D;
+                    dst[i] = __bfloat16_as_ushort(__float2bfloat16_rn(y1));
+                    dst[i + half] = __bfloat16_as_ushort(__float2bfloat16_rn(y2));
+                }
+            } else {
+                const int j = (int)(u - n_pairs);
+                float a, unused;
+                dot_rows<false, 16>(p.W + ((int64_t)(Hq + Hkv) * D + j) * K, nullptr, act, K, lane, a, unused);
+                if (lane == 0) {
+                    const float v = __bfloat162float(__float2bfloat16_rn(a));
+                    p.v_layer[(int64_t)pos * Hkv * D + j] = __half_as_ushort(__float2half_rn(v));
+                }
+            }
+        }
+    } else {
+        for (int64_t n = first; n < p.N; n += warps) {
+            float a, b;
+            if constexpr (MODE == GEMV_SWIGLU) {
+                dot_rows<true, 8>(p.W + n * K, p.W2 + n * K, act, K, lane, a, b);
+                if (lane == 0) p.y_bf16[n] = __bfloat16_as_ushort(__float2bfloat16_rn(a / (1.0f + __expf(-a)) * b));
+            } else {
+                dot_rows<false, 16>(p.W + n * K, nullptr, act, K, lane, a, b);
+                if (lane == 0) p.y_f32[n] += a;
+            }
+        }
     }
 }
 
@@ -180,11 +235,10 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
     int64_t end = start + KVB_DECODE_KEYS_PER_SPLIT;
     if (end > (int64_t)pos + 1) end = (int64_t)pos + 1;
 
-    float qv[G][DPL];
-#pragma unroll
-    for (int h = 0; h < G; ++h)
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) qv[h][e] = bf16_to_f(q[(g * G + h) * D + lane * DPL + e]);
+    // q of the G heads in shared memory (registers go to the K/V prefetch)
+    __shared__ __align__(16) float qs[G][D];
+    for (int i = threadIdx.x; i < G * D; i += ATT_THREADS) qs[i / D][i % D] = bf16_to_f(q[(g * G) * D + i]);
+    __syncthreads();
     float o[G][DPL];
 #pragma unroll
     for (int h = 0; h < G; ++h)
@@ -220,9 +274,17 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
             for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
 #pragma unroll
             for (int h = 0; h < G; ++h) {
+                float qv[DPL];
+                if constexpr (DPL == 4) {
+                    const float4 t4 = *reinterpret_cast<const float4*>(&qs[h][lane * 4]);
+                    qv[0] = t4.x; qv[1] = t4.y; qv[2] = t4.z; qv[3] = t4.w;
+                } else {
+                    const float2 t2 = *reinterpret_cast<const float2*>(&qs[h][lane * 2]);
+                    qv[0] = t2.x; qv[1] = t2.y;
+                }
                 float acc = 0.f;
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[e], acc);
+                for (int e = 0; e < DPL; ++e) acc = fmaf(qv[e], kf[e], acc);
                 sc[k * G + h] = acc;
             }
         }
@@ -302,13 +364,13 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
 
 // One block per q head: COMB_GROUPS groups of D threads, each over every COMB_GROUPS-th CTA
 // partial, then merged in shared memory.
-constexpr int COMB_GROUPS = 4;
+constexpr int COMB_GROUPS = 8;
 __global__ void decode_combine_kernel(const float* __restrict__ pm, const float* __restrict__ pl,
                                       const float* __restrict__ po, const int32_t* __restrict__ pos_ptr,
                                       int64_t max_pos, int keys_per_block, int Hq, int D, uint16_t* __restrict__ out,
                                       int* status) {
     __shared__ float s_m[COMB_GROUPS], s_l[COMB_GROUPS];
-    __shared__ float s_o[COMB_GROUPS][128];
+    __shared__ float s_o[COMB_GROUPS][128];   // D <= 128
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
     const int hq = blockIdx.x, d = threadIdx.x % D, grp = threadIdx.x / D;
@@ -369,17 +431,19 @@ kvb_status launch_decode_embed(const uint16_t* embed, const int32_t* tokens, con
     return cuda_ok(cudaGetLastError(), "decode embed launch");
 }
 
-kvb_status launch_gemv(int mode, const uint16_t* W, const uint16_t* W2, int64_t N, int K, const uint16_t* a,
-                       float* y_f32, uint16_t* y_bf16, cudaStream_t st) {
-    if (N <= 0) return KVB_OK;
-    if (K <= 0 || K % 8 || K > KVB_DECODE_MAX_K)
-        return fail(KVB_ERR_UNSUPPORTED, "gemv: K = %d must be a positive multiple of 8 up to %d", K, KVB_DECODE_MAX_K);
-    const size_t smem = (size_t)K * sizeof(float);
+kvb_status launch_gemv(int mode, const GemvArgs& p, cudaStream_t st) {
+    if (p.K <= 0 || p.K % 8 || p.K > KVB_DECODE_MAX_K)
+        return fail(KVB_ERR_UNSUPPORTED, "gemv: K = %d must be a positive multiple of 8 up to %d", p.K,
+                    KVB_DECODE_MAX_K);
+    const size_t smem = (size_t)p.K * sizeof(uint16_t);
     static bool attr[3] = {false, false, false};
-    auto set = [&](auto kern) -> kvb_status {
+    int64_t units = p.N;
+    if (mode == GEMV_QKV) units = (int64_t)(p.Hq + p.Hkv) * (p.D / 2) + (int64_t)p.Hkv * p.D;
+    if (units <= 0) return KVB_OK;
+    auto go = [&](auto kern) -> kvb_status {
         if (!attr[mode]) {
             kvb_status s = cuda_ok(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        KVB_DECODE_MAX_K * (int)sizeof(float)),
+                                                        KVB_DECODE_MAX_K * (int)sizeof(uint16_t)),
                                    "gemv smem");
             if (s != KVB_OK) return s;
             attr[mode] = true;
@@ -388,33 +452,23 @@ kvb_status launch_gemv(int mode, const uint16_t* W, const uint16_t* W2, int64_t 
         kvb_status s = cuda_ok(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, GEMV_THREADS, smem),
                                "gemv occupancy");
         if (s != KVB_OK) return s;
-        int64_t blocks = (N + GEMV_THREADS / 32 - 1) / (GEMV_THREADS / 32);
+        int64_t blocks = (units + GEMV_THREADS / 32 - 1) / (GEMV_THREADS / 32);
         const int64_t cap = (int64_t)num_sms() * (per_sm > 0 ? per_sm : 1);
         if (blocks > cap) blocks = cap;
-        kern<<<(unsigned)blocks, GEMV_THREADS, smem, st>>>(W, W2, N, K, a, y_f32, y_bf16);
+        kern<<<(unsigned)blocks, GEMV_THREADS, smem, st>>>(p);
         count_launch();
         return cuda_ok(cudaGetLastError(), "gemv launch");
     };
     switch (mode) {
-        case GEMV_F32: return set(gemv_kernel<GEMV_F32>);
-        case GEMV_RESID: return set(gemv_kernel<GEMV_RESID>);
-        case GEMV_SWIGLU: return set(gemv_kernel<GEMV_SWIGLU>);
+        case GEMV_QKV: return go(gemv_kernel<GEMV_QKV>);
+        case GEMV_RESID: return go(gemv_kernel<GEMV_RESID>);
+        case GEMV_SWIGLU: return go(gemv_kernel<GEMV_SWIGLU>);
         default: return fail(KVB_ERR_INVALID_ARG, "gemv: unknown mode %d", mode);
     }
 }
 
-kvb_status launch_qkv_finish(const float* qkv, const int32_t* pos, int64_t max_pos, const float* cos_t,
-                             const float* sin_t, int D, int Hq, int Hkv, uint16_t* q_out, uint16_t* k_layer,
-                             uint16_t* v_layer, int* status, cudaStream_t st) {
-    const int n = (Hq + Hkv) * (D / 2) + Hkv * D;
-    qkv_finish_kernel<<<(n + 255) / 256, 256, 0, st>>>(qkv, pos, max_pos, cos_t, sin_t, D, Hq, Hkv, q_out, k_layer,
-                                                       v_layer, status);
-    count_launch();
-    return cuda_ok(cudaGetLastError(), "qkv finish launch");
-}
-
 // CTA partials of the decode attention for positions below max_pos
-int decode_splits(int64_t max_pos) {
+int decode_splits(int64_t max_pos, int) {
     const int64_t per_block = (int64_t)KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32);
     return (int)((max_pos + per_block - 1) / per_block);
 }
@@ -423,7 +477,7 @@ kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint1
                               const int32_t* pos, int64_t max_pos, float sl2, float* pm, float* pl, float* po,
                               uint16_t* out, int* status, cudaStream_t st) {
     const int G = Hq / Hkv;
-    const int n_splits = decode_splits(max_pos);
+    const int n_splits = decode_splits(max_pos, Hkv);
     kvb_status s;
     if (D == 128 && G == 4) s = run_attn<128, 4>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
     else if (D == 128 && G == 8) s = run_attn<128, 8>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);

@@ -106,15 +106,30 @@ kvb_status launch_deviation_histogram(const uint16_t* ka, int64_t lda, const uin
 // ---------------------------------------------------------------- greedy decode
 constexpr int KVB_DECODE_KEYS_PER_SPLIT = 128;   // cache rows per warp split of the decode attention
 constexpr int KVB_DECODE_MAX_K = 16384;          // longest input row of a decode GEMV (shared memory)
-enum GemvMode { GEMV_F32 = 0, GEMV_RESID = 1, GEMV_SWIGLU = 2 };
-int decode_splits(int64_t max_pos);
+enum GemvMode { GEMV_QKV = 0, GEMV_RESID = 1, GEMV_SWIGLU = 2 };
+struct GemvArgs {
+    const uint16_t* W;            // [N][K] bf16 (QKV: w_qkv; SwiGLU: gate rows)
+    const uint16_t* W2;           // SwiGLU: up rows [N][K]
+    int64_t N;                    // output rows (RESID, SWIGLU)
+    int K;
+    const uint16_t* a;            // RESID: bf16 input row [K]
+    const float* x;               // QKV, SWIGLU: fp32 residual row [K] (RMSNorm prologue)
+    const float* g;               // its RMSNorm gain [K]
+    float eps;
+    float* y_f32;                 // RESID: x += y
+    uint16_t* y_bf16;             // SWIGLU: h (bf16 [N])
+    const int32_t* pos;           // QKV: position (device), 0 <= pos < max_pos
+    int64_t max_pos;
+    const float *cos_t, *sin_t;   // QKV: RoPE tables [max_pos][D/2]
+    int D, Hq, Hkv;
+    uint16_t* q_out;              // QKV: bf16 [Hq][D]
+    uint16_t *k_layer, *v_layer;  // QKV: this layer's cache [n_rows][Hkv][D]
+    int* status;
+};
+int decode_splits(int64_t max_pos, int Hkv);
 kvb_status launch_decode_embed(const uint16_t* embed, const int32_t* tokens, const int32_t* pos, int64_t max_pos,
                                int64_t vocab, int H, float* x, int* status, cudaStream_t st);
-kvb_status launch_gemv(int mode, const uint16_t* W, const uint16_t* W2, int64_t N, int K, const uint16_t* a,
-                       float* y_f32, uint16_t* y_bf16, cudaStream_t st);
-kvb_status launch_qkv_finish(const float* qkv, const int32_t* pos, int64_t max_pos, const float* cos_t,
-                             const float* sin_t, int D, int Hq, int Hkv, uint16_t* q_out, uint16_t* k_layer,
-                             uint16_t* v_layer, int* status, cudaStream_t st);
+kvb_status launch_gemv(int mode, const GemvArgs& p, cudaStream_t st);
 kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hq, int Hkv, int D,
                               const int32_t* pos, int64_t max_pos, float sl2, float* pm, float* pl, float* po,
                               uint16_t* out, int* status, cudaStream_t st);
