@@ -237,6 +237,8 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
 
     // q of the G heads in shared memory (registers go to the K/V prefetch)
     __shared__ __align__(16) float qs[G][D];
+    __shared__ __align__(16) float sp[ATT_THREADS / 32][32];   // per warp: this step's weights
+    __shared__ float sa[ATT_THREADS / 32][G];                   // per warp: rescale factor per head
     for (int i = threadIdx.x; i < G * D; i += ATT_THREADS) qs[i / D][i % D] = bf16_to_f(q[(g * G) * D + i]);
     __syncthreads();
     float o[G][DPL];
@@ -267,25 +269,30 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
         // loads of the next step go out before this step's arithmetic
         if (k0 + KS < end) fetch(k0 + KS, nk, nv);
         float sc[32];
-#pragma unroll
-        for (int k = 0; k < KS; ++k) {
-            float kf[DPL];
-#pragma unroll
-            for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
+        {
+            float qv[G][DPL];   // this lane's head dims of q, once per step
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                float qv[DPL];
                 if constexpr (DPL == 4) {
                     const float4 t4 = *reinterpret_cast<const float4*>(&qs[h][lane * 4]);
-                    qv[0] = t4.x; qv[1] = t4.y; qv[2] = t4.z; qv[3] = t4.w;
+                    qv[h][0] = t4.x; qv[h][1] = t4.y; qv[h][2] = t4.z; qv[h][3] = t4.w;
                 } else {
                     const float2 t2 = *reinterpret_cast<const float2*>(&qs[h][lane * 2]);
-                    qv[0] = t2.x; qv[1] = t2.y;
+                    qv[h][0] = t2.x; qv[h][1] = t2.y;
                 }
-                float acc = 0.f;
+            }
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) acc = fmaf(qv[e], kf[e], acc);
-                sc[k * G + h] = acc;
+            for (int k = 0; k < KS; ++k) {
+                float kf[DPL];
+#pragma unroll
+                for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    float acc = 0.f;
+#pragma unroll
+                    for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[e], acc);
+                    sc[k * G + h] = acc;
+                }
             }
         }
         // reduce-scatter: afterwards lane L holds the full dot product of index L
@@ -306,16 +313,21 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
 #pragma unroll
         for (int off = G; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
         const float m_new = fmaxf(m_run, mx);
-        const float alpha = (m_new == -INFINITY) ? 1.f : exp2f(m_run - m_new);
-        const float pv = (t == -INFINITY) ? 0.f : exp2f(t - m_new);
+        const float alpha = (m_new == -INFINITY) ? 1.f : fast_exp2(m_run - m_new);
+        const float pv = (t == -INFINITY) ? 0.f : fast_exp2(t - m_new);
         float ps = pv;
 #pragma unroll
         for (int off = G; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
         l_run = l_run * alpha + ps;
         m_run = m_new;
+        // this step's weights (index key * G + head) and the heads' rescale factors to every lane
+        __syncwarp();
+        sp[warp][lane] = pv;
+        if (lane < G) sa[warp][lane] = alpha;
+        __syncwarp();
 #pragma unroll
         for (int h = 0; h < G; ++h) {
-            const float ah = __shfl_sync(0xffffffffu, alpha, h);
+            const float ah = sa[warp][h];
 #pragma unroll
             for (int e = 0; e < DPL; ++e) o[h][e] *= ah;
         }
@@ -328,10 +340,23 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
                 vf[2 * i] = f.x; vf[2 * i + 1] = f.y;
             }
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const float pk = __shfl_sync(0xffffffffu, pv, k * G + h);
+            float pk[G];   // weights of key k for the G heads, vector loads (broadcast)
+            if constexpr (G % 4 == 0) {
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk, vf[e], o[h][e]);
+                for (int h4 = 0; h4 < G; h4 += 4) {
+                    const float4 t = *reinterpret_cast<const float4*>(&sp[warp][k * G + h4]);
+                    pk[h4] = t.x; pk[h4 + 1] = t.y; pk[h4 + 2] = t.z; pk[h4 + 3] = t.w;
+                }
+            } else {
+#pragma unroll
+                for (int h2 = 0; h2 < G; h2 += 2) {
+                    const float2 t = *reinterpret_cast<const float2*>(&sp[warp][k * G + h2]);
+                    pk[h2] = t.x; pk[h2 + 1] = t.y;
+                }
+            }
+            for (int h = 0; h < G; ++h) {
+#pragma unroll
+                for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk[h], vf[e], o[h][e]);
             }
         }
 #pragma unroll
