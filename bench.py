@@ -71,6 +71,23 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The slowest replica's step time: max over the ranks of the process group (the
+    replicas share nothing else, so this is the only collective of the benchmark)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_tokens_per_s(n_tokens: int, world: int, ms: float) -> float:
+    """Whole-job throughput of `world` replicas that each prefill `n_tokens` in `ms`."""
+    return world * n_tokens / (ms * 1e-3)
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -268,10 +285,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
     barrier()
     clk = clocks.stop()
     ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, dev)
     assert kvb.device_status(ws) == 0, "device wait timed out"
 
     # algorithmic work of the step (from the chosen rows, read back after the timed region)
@@ -451,7 +465,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
                        "n_ctx": n_ctx, "n_query": nq, "n_tokens": N, "r": r, "k": k, "check_layer": 1,
                        "l2": "inputs larger than L2 (16.3 GB of chunk KV caches read per step)",
                        "parallelism": f"replicas x{world}"},
-            "tokens_per_s": round(world * N / (ms * 1e-3), 1),
+            "tokens_per_s": round(replica_tokens_per_s(N, world, ms), 1),
             "r1_dense": r1,
             "ttft_reduction_vs_r1": (round(1.0 - ms / r1["ttft_ms"], 4) if r1 else None),
             "algorithmic_tflops": round(total_flop / (ms * 1e-3) / 1e12, 2),
