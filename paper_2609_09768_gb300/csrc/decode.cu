@@ -387,31 +387,30 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
     }
 }
 
-// One block per q head: COMB_GROUPS groups of D threads, each over every COMB_GROUPS-th CTA
-// partial, then merged in shared memory.
-constexpr int COMB_GROUPS = 8;
-__global__ void decode_combine_kernel(const float* __restrict__ pm, const float* __restrict__ pl,
-                                      const float* __restrict__ po, const int32_t* __restrict__ pos_ptr,
-                                      int64_t max_pos, int keys_per_block, int Hq, int D, uint16_t* __restrict__ out,
-                                      int* status) {
+// Block (q head, 32 head dims): COMB_GROUPS groups of 32 threads, group q over CTA partials
+// q, q + COMB_GROUPS, ..., then merged in shared memory.
+constexpr int COMB_GROUPS = 32;
+__global__ void __launch_bounds__(32 * COMB_GROUPS)
+decode_combine_kernel(const float* __restrict__ pm, const float* __restrict__ pl, const float* __restrict__ po,
+                      const int32_t* __restrict__ pos_ptr, int64_t max_pos, int keys_per_block, int Hq, int D,
+                      uint16_t* __restrict__ out, int* status) {
     __shared__ float s_m[COMB_GROUPS], s_l[COMB_GROUPS];
-    __shared__ float s_o[COMB_GROUPS][128];   // D <= 128
+    __shared__ float s_o[COMB_GROUPS][32];
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
-    const int hq = blockIdx.x, d = threadIdx.x % D, grp = threadIdx.x / D;
+    const int hq = blockIdx.x, d = blockIdx.y * 32 + (threadIdx.x & 31), grp = threadIdx.x >> 5;
     const int n = (pos + keys_per_block) / keys_per_block;   // CTA partials holding keys [0, pos]
     float M = -INFINITY;
     for (int s = grp; s < n; s += COMB_GROUPS) M = fmaxf(M, pm[(int64_t)s * Hq + hq]);
     float L = 0.f, O = 0.f;
-#pragma unroll 4
     for (int s = grp; s < n; s += COMB_GROUPS) {
         const float ms = pm[(int64_t)s * Hq + hq];
         const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
         L += w * pl[(int64_t)s * Hq + hq];
         O += w * po[((int64_t)s * Hq + hq) * D + d];
     }
-    if (d == 0) { s_m[grp] = M; s_l[grp] = L; }
-    s_o[grp][d] = O;
+    if ((threadIdx.x & 31) == 0) { s_m[grp] = M; s_l[grp] = L; }
+    s_o[grp][threadIdx.x & 31] = O;
     __syncthreads();
     if (grp == 0) {
         float MM = -INFINITY;
@@ -422,7 +421,7 @@ __global__ void decode_combine_kernel(const float* __restrict__ pm, const float*
         for (int q2 = 0; q2 < COMB_GROUPS; ++q2) {
             const float w = (s_m[q2] == -INFINITY) ? 0.f : exp2f(s_m[q2] - MM);
             LL += w * s_l[q2];
-            OO += w * s_o[q2][d];
+            OO += w * s_o[q2][threadIdx.x];
         }
         out[hq * D + d] = __bfloat16_as_ushort(__float2bfloat16_rn(LL > 0.f ? OO / LL : 0.f));
     }
@@ -511,7 +510,7 @@ kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint1
     else if (D == 64 && G == 4) s = run_attn<64, 4>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
     else return fail(KVB_ERR_UNSUPPORTED, "decode attention: head_dim %d with %d q heads per kv head not built", D, G);
     if (s != KVB_OK) return s;
-    decode_combine_kernel<<<(unsigned)Hq, (unsigned)(D * COMB_GROUPS), 0, st>>>(
+    decode_combine_kernel<<<dim3((unsigned)Hq, (unsigned)(D / 32)), 32 * COMB_GROUPS, 0, st>>>(
         pm, pl, po, pos, max_pos, KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32), Hq, D, out, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode combine launch");

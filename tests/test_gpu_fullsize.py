@@ -259,3 +259,44 @@ def test_headline_pipelined_ingest_equals_device_resident(kvb, headline):
     assert kvb.device_status(wsp) == 0
     k = blend.num_selected(WL.r, N_CTX)
     assert torch.equal(fh, fh2) and torch.equal(sel[:k], sel2[:k]) and torch.equal(ck, ck2) and torch.equal(cv, cv2)
+
+
+def test_headline_decode_step_appends_the_dense_prefill_row(kvb, headline):
+    """One greedy decode step after the 124k selective prefill: it writes the new token's
+    K/V into row N of every layer and nothing else; layer 0's appended row (which depends
+    only on the token and its position) equals the dense prefill of the N + 1 tokens at row
+    N within one bf16 ulp; the next token is a valid id and pos advances."""
+    h = headline
+    cap = N + 2
+    cfg = h["cfg"]
+    rope = kvb.RopeTable(cfg, cap)
+    L = SHAPE.n_layers
+    ck = torch.zeros(L, cap, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
+    cv = torch.zeros(ck.shape, dtype=torch.float16, device="cuda")
+    fh, _, _ = kvb.selective_prefill(cfg, h["model"], rope, h["kch"], h["vch"], ck, cv, h["toks"], h["dstarts"],
+                                     N_CTX, WL.n_query, WL.r, 1, ws=h["ws"])
+    lm = synth.make_lm_head(SHAPE, 0, "cuda")
+    first, _ = kvb.lm_head_argmax(cfg, lm, fh[WL.n_query - 1:].contiguous())
+    tokens = torch.zeros(cap + 1, dtype=torch.int32, device="cuda")
+    tokens[:N] = h["toks"]
+    tokens[N:N + 1] = first
+    before_k = ck[:, :N].clone()
+    pos = torch.tensor([N], dtype=torch.int32, device="cuda")
+    dws = kvb.decode_workspace(cfg, cap)
+    kvb.decode_step(cfg, h["model"], rope, ck, cv, lm, tokens, pos, cap, ws=dws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(dws) == 0 and int(pos.item()) == N + 1
+    nxt = int(tokens[N + 1].item())
+    assert 0 <= nxt < SHAPE.vocab
+    assert torch.equal(ck[:, :N], before_k)
+    assert torch.count_nonzero(ck[:, N + 1:]) == 0
+    assert torch.all(ck[:, N].abs().sum(dim=(-1, -2)) > 0)
+    # layer 0 of the dense prefill of the same N + 1 tokens, row N
+    kd = torch.zeros(L, N + 1, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
+    vd = torch.zeros(kd.shape, dtype=torch.float16, device="cuda")
+    wsd = kvb.workspace(cfg, N + 1)
+    kvb.full_prefill(cfg, h["model"], rope, kd, vd, tokens[:N + 1].contiguous(), ws=wsd)
+    torch.cuda.synchronize()
+    assert kvb.device_status(wsd) == 0
+    assert_close_bf16(ck[0, N].cpu(), np64(kd[0, N].cpu()), "decode layer-0 K row vs dense prefill")
+    assert_close_bf16(cv[0, N].cpu(), np64(vd[0, N].cpu()), "decode layer-0 V row vs dense prefill")
