@@ -95,6 +95,17 @@ kvb_status make_tmap_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t 
     return KVB_OK;
 }
 
+kvb_status ensure_smem_limit(const void* kernel, int bytes, std::atomic<uint64_t>& done, const char* what) {
+    int dev = 0;
+    kvb_status s = cuda_ok(cudaGetDevice(&dev), what);
+    if (s != KVB_OK) return s;
+    const uint64_t bit = 1ull << (dev & 63);
+    if (done.load(std::memory_order_acquire) & bit) return KVB_OK;
+    s = cuda_ok(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes), what);
+    if (s == KVB_OK) done.fetch_or(bit, std::memory_order_release);
+    return s;
+}
+
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 size_t workspace_layout(const kvb_config* c, int64_t n, void* base, Workspace* w) {

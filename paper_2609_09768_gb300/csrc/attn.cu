@@ -343,14 +343,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
 template <int D>
 kvb_status run(const uint16_t* q, const CUtensorMap& k, const CUtensorMap& v, const AttnParams& p, int nb,
                cudaStream_t st) {
-    static bool attr_set = false;
+    static std::atomic<uint64_t> smem_set{0};
     auto kern = attn_kernel<D>;
-    if (!attr_set) {
-        kvb_status s = cuda_ok(
-            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<D>::TOTAL), "attn smem");
-        if (s != KVB_OK) return s;
-        attr_set = true;
-    }
+    kvb_status s = ensure_smem_limit((const void*)kern, Smem<D>::TOTAL, smem_set, "attn smem");
+    if (s != KVB_OK) return s;
     const int64_t grid = (int64_t)nb * p.Hkv;
     kern<<<(unsigned)grid, THREADS, Smem<D>::TOTAL, st>>>(q, k, v, p, nb);
     count_launch();

@@ -460,20 +460,16 @@ kvb_status launch_gemv(int mode, const GemvArgs& p, cudaStream_t st) {
         return fail(KVB_ERR_UNSUPPORTED, "gemv: K = %d must be a positive multiple of 8 up to %d", p.K,
                     KVB_DECODE_MAX_K);
     const size_t smem = (size_t)p.K * sizeof(uint16_t);
-    static bool attr[3] = {false, false, false};
+    static std::atomic<uint64_t> smem_set[3];
     int64_t units = p.N;
     if (mode == GEMV_QKV) units = (int64_t)(p.Hq + p.Hkv) * (p.D / 2) + (int64_t)p.Hkv * p.D;
     if (units <= 0) return KVB_OK;
     auto go = [&](auto kern) -> kvb_status {
-        if (!attr[mode]) {
-            kvb_status s = cuda_ok(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        KVB_DECODE_MAX_K * (int)sizeof(uint16_t)),
-                                   "gemv smem");
-            if (s != KVB_OK) return s;
-            attr[mode] = true;
-        }
+        kvb_status s = ensure_smem_limit((const void*)kern, KVB_DECODE_MAX_K * (int)sizeof(uint16_t), smem_set[mode],
+                                         "gemv smem");
+        if (s != KVB_OK) return s;
         int per_sm = 0;
-        kvb_status s = cuda_ok(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, GEMV_THREADS, smem),
+        s = cuda_ok(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, GEMV_THREADS, smem),
                                "gemv occupancy");
         if (s != KVB_OK) return s;
         int64_t blocks = (units + GEMV_THREADS / 32 - 1) / (GEMV_THREADS / 32);

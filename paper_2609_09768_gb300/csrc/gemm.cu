@@ -298,14 +298,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
 template <int EPI, int HD>
 kvb_status run(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& b2, const GemmParams& p, int tiles,
                cudaStream_t st) {
-    static bool attr_set = false;
+    static std::atomic<uint64_t> smem_set{0};
     auto kern = gemm_kernel<EPI, HD>;
-    if (!attr_set) {
-        kvb_status s = cuda_ok(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES),
-                               "gemm smem attribute");
-        if (s != KVB_OK) return s;
-        attr_set = true;
-    }
+    kvb_status s = ensure_smem_limit((const void*)kern, SMEM_BYTES, smem_set, "gemm smem attribute");
+    if (s != KVB_OK) return s;
     const int grid = tiles < num_sms() ? tiles : num_sms();
     kern<<<grid, THREADS, SMEM_BYTES, st>>>(a, b, b2, p);
     count_launch();

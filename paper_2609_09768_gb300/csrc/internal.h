@@ -1,6 +1,8 @@
 // Host-side internals shared by the translation units of libkvblend.
 #pragma once
 
+#include <atomic>
+
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -13,6 +15,10 @@ namespace kvb {
 kvb_status fail(kvb_status s, const char* fmt, ...);
 // KVB_OK, or KVB_ERR_CUDA with the CUDA error text.
 kvb_status cuda_ok(cudaError_t e, const char* what);
+// Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current device the first time
+// it is needed there (the attribute is per device); `done` is the caller's per-kernel mask of
+// devices already set.  Thread-safe: a race only repeats the idempotent call.
+kvb_status ensure_smem_limit(const void* kernel, int bytes, std::atomic<uint64_t>& done, const char* what);
 int num_sms();
 // Counts kernels the library launched (for the prefill's launch report).
 void count_launch();

@@ -98,14 +98,9 @@ kvb_status launch_lmhead(const uint16_t* W, int64_t vocab, int H, const float* x
     kvb_status s = cuda_ok(cudaMemsetAsync(keys, 0, (size_t)n * sizeof(unsigned long long), st), "lm head: clear keys");
     if (s != KVB_OK) return s;
     const size_t smem = (size_t)n * H * sizeof(float);
-    static bool attr = false;
-    if (!attr) {
-        s = cuda_ok(cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         KVB_LMHEAD_MAX_ROWS * 8192 * 4),
-                    "lm head smem");
-        if (s != KVB_OK) return s;
-        attr = true;
-    }
+    static std::atomic<uint64_t> smem_set{0};
+    s = ensure_smem_limit((const void*)lmhead_kernel, KVB_LMHEAD_MAX_ROWS * 8192 * 4, smem_set, "lm head smem");
+    if (s != KVB_OK) return s;
     // one wave of resident blocks, each warp striding over the vocabulary
     int per_sm = 0;
     s = cuda_ok(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_kernel, THREADS, smem), "lm head occupancy");
