@@ -14,8 +14,11 @@ prefill (all rows), the per-chunk isolated prefill (block-diagonal ranges) and
 the selective recompute of Sec. 3.2 (selected rows over the whole blended cache).
 
 RoPE is the rotate-half form used by Llama: dimension i is paired with i + D/2
-and the pair is rotated by angle pos * w_i, w_i = theta^(-2i/D), with Llama 3.1's
-frequency scaling (factor, low/high frequency factors, original context).
+and the pair is rotated by angle pos * w_i, w_i = theta^(-2i/D), with one of two
+frequency scalings: Llama 3.1's (factor, low/high frequency factors, original
+context), or YaRN's, which the paper's second model (Qwen2.5-7B-Instruct, Sec. 4)
+uses.  YaRN also divides the attention logits by a temperature.  The q/k/v
+projections may carry an additive bias (the layer dict's optional "b_qkv").
 
 Precision.  Arithmetic is float64.  Sec. 4 of the paper states that the model's
 computations run in bfloat16 (only the position adjustment in float32).  With
@@ -41,6 +44,9 @@ import numpy as np
 
 F64 = np.float64
 
+# frequency scaling of the rotary embedding
+ROPE_PLAIN, ROPE_LLAMA3, ROPE_YARN = 0, 1, 2
+
 
 @dataclass(frozen=True)
 class Shape:
@@ -51,7 +57,7 @@ class Shape:
     mlp_dim: int
     rms_eps: float
     rope_theta: float
-    rope_llama3: bool = False
+    rope_scaling: int = ROPE_PLAIN
     rs_factor: float = 8.0
     rs_low: float = 1.0
     rs_high: float = 4.0
@@ -63,7 +69,7 @@ class Shape:
     def of(s, act_bf16: bool = False, accum32: bool = False) -> "Shape":
         """Copy the fields from any object that has them (e.g. a ModelShape)."""
         return Shape(s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.mlp_dim,
-                     float(s.rms_eps), float(s.rope_theta), bool(s.rope_llama3),
+                     float(s.rms_eps), float(s.rope_theta), int(s.rope_scaling),
                      float(s.rs_factor), float(s.rs_low), float(s.rs_high), int(s.rs_orig_ctx), act_bf16,
                      accum32)
 
@@ -93,19 +99,23 @@ def act(s: "Shape", x: np.ndarray) -> np.ndarray:
 # ----------------------------------------------------------------------------- RoPE
 
 def rope_inv_freq(s: Shape) -> np.ndarray:
-    """w_i = theta^(-2i/D), i < D/2, then Llama 3.1 frequency scaling.
+    """w_i = theta^(-2i/D), i < D/2, then the shape's frequency scaling.
 
-    Scaling (from the public Llama 3.1 model definition): with wavelength
+    Llama 3.1 scaling (from the public Llama 3.1 model definition): with wavelength
     lam = 2*pi/w, frequencies whose wavelength is shorter than orig/high are
     kept; those longer than orig/low are divided by `factor`; in between the
     two are blended with s = (orig/lam - low)/(high - low):
         w' = (1 - s) * w / factor + s * w.
+    YaRN scaling: `yarn_inv_freq`.
     """
+    if s.rope_scaling == ROPE_YARN:
+        return yarn_inv_freq(s)
     D = s.head_dim
     i = np.arange(D // 2, dtype=F64)
     w = s.rope_theta ** (-(2.0 * i) / D)
-    if not s.rope_llama3:
+    if s.rope_scaling == ROPE_PLAIN:
         return w
+    assert s.rope_scaling == ROPE_LLAMA3, s.rope_scaling
     out = np.empty_like(w)
     lo_wavelen = s.rs_orig_ctx / s.rs_low     # longest wavelength still blended
     hi_wavelen = s.rs_orig_ctx / s.rs_high    # shortest wavelength blended
@@ -119,6 +129,48 @@ def rope_inv_freq(s: Shape) -> np.ndarray:
             sm = (s.rs_orig_ctx / lam - s.rs_low) / (s.rs_high - s.rs_low)
             out[j] = (1.0 - sm) * w[j] / s.rs_factor + sm * w[j]
     return out
+
+
+def yarn_inv_freq(s: Shape) -> np.ndarray:
+    """YaRN's "NTK-by-parts" interpolation (Peng et al., YaRN, Sec. 3.2), in that
+    paper's notation, with s.rs_factor = s, s.rs_low = alpha, s.rs_high = beta and
+    s.rs_orig_ctx = L (the context length the model was trained at):
+
+        theta_d  = b^(-2d/|D|)               frequency of rotation pair d
+        lambda_d = 2 pi / theta_d            its wavelength in tokens
+        r(d)     = L / lambda_d              turns it makes over the original context
+        gamma(r) = 0 if r < alpha, 1 if r > beta, (r - alpha)/(beta - alpha) otherwise
+        h(theta_d) = (1 - gamma(r(d))) theta_d / s + gamma(r(d)) theta_d
+
+    Pairs that turn fewer than alpha times over L are interpolated by s (position
+    interpolation), pairs that turn more than beta times are left alone, and the
+    ramp is linear in r between them."""
+    D = s.head_dim
+    L, scale, alpha, beta = float(s.rs_orig_ctx), float(s.rs_factor), float(s.rs_low), float(s.rs_high)
+    out = np.empty(D // 2, dtype=F64)
+    for d in range(D // 2):
+        theta = s.rope_theta ** (-2.0 * d / D)
+        lam = 2.0 * math.pi / theta
+        r = L / lam
+        if r < alpha:
+            gamma = 0.0
+        elif r > beta:
+            gamma = 1.0
+        else:
+            gamma = (r - alpha) / (beta - alpha)
+        out[d] = (1.0 - gamma) * theta / scale + gamma * theta
+    return out
+
+
+def logit_scale(s: Shape) -> float:
+    """Factor applied to q.k before the softmax: 1/sqrt(D).  YaRN (Sec. 3.4 of its
+    paper) also divides the logits by a temperature t with sqrt(1/t) = 0.1 ln(s) + 1,
+    i.e. multiplies them by (0.1 ln(s) + 1)^2."""
+    base = 1.0 / math.sqrt(s.head_dim)
+    if s.rope_scaling == ROPE_YARN:
+        m = 0.1 * math.log(s.rs_factor) + 1.0
+        return base * m * m
+    return base
 
 
 def rope_cos_sin(s: Shape, pos) -> tuple[np.ndarray, np.ndarray]:
@@ -170,8 +222,9 @@ def attention_rows(s: Shape, q: np.ndarray, k_cache: np.ndarray, v_cache: np.nda
     row_lo:   [m] first cache row it may read (None: 0)
     returns   [m, Hq, D]
 
-    out[r, j] = sum_t softmax_t(q[r,j] . k[t, g] / sqrt(D)) v[t, g] over lo_r <= t <= hi_r,
-    g = j // (Hq / Hkv); softmax taken with max subtraction.
+    out[r, j] = sum_t softmax_t(c * q[r,j] . k[t, g]) v[t, g] over lo_r <= t <= hi_r,
+    g = j // (Hq / Hkv), c = logit_scale(s) (1/sqrt(D) without YaRN); softmax taken
+    with max subtraction.
     """
     m, Hq, D = q.shape
     Hkv = k_cache.shape[1]
@@ -179,7 +232,7 @@ def attention_rows(s: Shape, q: np.ndarray, k_cache: np.ndarray, v_cache: np.nda
     row_hi = np.asarray(row_hi, dtype=np.int64)
     row_lo = np.zeros(m, dtype=np.int64) if row_lo is None else np.asarray(row_lo, dtype=np.int64)
     out = np.zeros((m, Hq, D), dtype=F64)
-    scale = 1.0 / math.sqrt(D)
+    scale = logit_scale(s)
     for r0 in range(0, m, block):
         r1 = min(m, r0 + block)
         lo, hi = row_lo[r0:r1], row_hi[r0:r1]
@@ -201,10 +254,12 @@ def attention_rows(s: Shape, q: np.ndarray, k_cache: np.ndarray, v_cache: np.nda
 
 
 def qkv_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> tuple[np.ndarray, np.ndarray, np.ndarray]:
-    """RMSNorm -> QKV projection -> RoPE at `rope_pos`.  Returns q [m,Hq,D], k, v [m,Hkv,D]."""
+    """RMSNorm -> QKV projection (+ bias) -> RoPE at `rope_pos`.  Returns q [m,Hq,D], k, v [m,Hkv,D]."""
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
     n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
     qkv = linear(n1, lw["w_qkv"], s.accum32)
+    if lw.get("b_qkv") is not None:
+        qkv = qkv + as64(lw["b_qkv"])
     m = x.shape[0]
     q = qkv[:, : Hq * D].reshape(m, Hq, D)
     k = qkv[:, Hq * D: (Hq + Hkv) * D].reshape(m, Hkv, D)
@@ -214,11 +269,14 @@ def qkv_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> tuple[np.ndarray, n
 
 
 def k_rows(s: Shape, lw: dict, x: np.ndarray, rope_pos) -> np.ndarray:
-    """Only the key projection (RMSNorm -> W_k -> RoPE), [m, Hkv, D]."""
+    """Only the key projection (RMSNorm -> W_k (+ bias) -> RoPE), [m, Hkv, D]."""
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
     n1 = act(s, rmsnorm(x, lw["attn_norm"], s.rms_eps))
     wk = as64(lw["w_qkv"])[Hq * D: (Hq + Hkv) * D]
-    k = linear(n1, wk, s.accum32).reshape(x.shape[0], Hkv, D)
+    k = linear(n1, wk, s.accum32)
+    if lw.get("b_qkv") is not None:
+        k = k + as64(lw["b_qkv"])[Hq * D: (Hq + Hkv) * D]
+    k = k.reshape(x.shape[0], Hkv, D)
     c, sn = rope_cos_sin(s, rope_pos)
     return act(s, apply_rope(k, c, sn))
 

@@ -155,7 +155,7 @@ def config(shape, n_layers: Optional[int] = None) -> Config:
     """kvb_config from any object with ModelShape's fields."""
     return Config(shape.hidden, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.mlp_dim,
                   shape.n_layers if n_layers is None else n_layers, shape.vocab, shape.rms_eps, shape.rope_theta,
-                  1 if shape.rope_llama3 else 0, shape.rs_factor, shape.rs_low, shape.rs_high, shape.rs_orig_ctx)
+                  int(shape.rope_scaling), shape.rs_factor, shape.rs_low, shape.rs_high, shape.rs_orig_ctx)
 
 
 # ---------------------------------------------------------------------------------- RoPE

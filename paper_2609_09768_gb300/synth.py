@@ -13,6 +13,7 @@ followed by the question):
 * embedding table: N(0, 1), rounded to bf16;
 * linear weights: N(0, 0.02), rounded to bf16 (so both sides read the same values);
 * RMSNorm gains: 1.0;
+* q/k/v projection bias (shapes that have one): N(0, 0.5^2), rounded to bf16, held as fp32;
 * chunks of equal length laid end to end, then a query suffix;
 * optionally two special tokens between consecutive documents (the last two ids of
   the vocabulary), whose rows of the concatenated cache are zero.
@@ -36,7 +37,12 @@ __all__ = [
 
 @dataclasses.dataclass(frozen=True)
 class ModelShape:
-    """Llama-3.1 decoder shape (hidden, heads, head dim, MLP dim, layers, RoPE)."""
+    """Decoder shape (hidden, heads, head dim, MLP dim, layers, RoPE).
+
+    rope_scaling: 0 plain RoPE, 1 Llama 3.1 frequency scaling (rs_factor, low/high
+    frequency factors rs_low/rs_high, original context rs_orig_ctx), 2 YaRN (scale
+    rs_factor, ramp bounds alpha = rs_low and beta = rs_high, original context
+    rs_orig_ctx).  qkv_bias: the q/k/v projections carry an additive bias."""
     hidden: int
     n_q_heads: int
     n_kv_heads: int
@@ -46,11 +52,12 @@ class ModelShape:
     vocab: int
     rms_eps: float = 1e-5
     rope_theta: float = 10000.0
-    rope_llama3: bool = False
+    rope_scaling: int = 0
     rs_factor: float = 8.0
     rs_low: float = 1.0
     rs_high: float = 4.0
     rs_orig_ctx: int = 8192
+    qkv_bias: bool = False
 
     @property
     def q_dim(self) -> int:
@@ -116,9 +123,21 @@ TINY = ModelShape(hidden=256, n_q_heads=4, n_kv_heads=2, head_dim=64, mlp_dim=68
                   n_layers=2, vocab=1024, rms_eps=1e-5, rope_theta=10000.0)
 LLAMA8B = ModelShape(hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128, mlp_dim=14336,
                      n_layers=32, vocab=128256, rms_eps=1e-5, rope_theta=500000.0,
-                     rope_llama3=True, rs_factor=8.0, rs_low=1.0, rs_high=4.0, rs_orig_ctx=8192)
+                     rope_scaling=1, rs_factor=8.0, rs_low=1.0, rs_high=4.0, rs_orig_ctx=8192)
+# Seven query heads per kv head, YaRN scaling (factor 4 over an original context shorter
+# than the workloads below, ramp between 1 and 32 turns) and a q/k/v bias: the features
+# of the paper's second model family, at sizes chosen here (not that model's own).
+YARN_GQA7_TINY = ModelShape(hidden=512, n_q_heads=7, n_kv_heads=1, head_dim=64, mlp_dim=1376,
+                            n_layers=2, vocab=1024, rms_eps=1e-6, rope_theta=1000000.0,
+                            rope_scaling=2, rs_factor=4.0, rs_low=1.0, rs_high=32.0, rs_orig_ctx=256,
+                            qkv_bias=True)
+YARN_GQA7 = ModelShape(hidden=1792, n_q_heads=14, n_kv_heads=2, head_dim=128, mlp_dim=4864,
+                       n_layers=2, vocab=32768, rms_eps=1e-6, rope_theta=1000000.0,
+                       rope_scaling=2, rs_factor=4.0, rs_low=1.0, rs_high=32.0, rs_orig_ctx=2048,
+                       qkv_bias=True)
 
-SHAPES: Dict[str, ModelShape] = {"tiny": TINY, "llama8b": LLAMA8B}
+SHAPES: Dict[str, ModelShape] = {"tiny": TINY, "llama8b": LLAMA8B, "yarn_gqa7_tiny": YARN_GQA7_TINY,
+                                 "yarn_gqa7": YARN_GQA7}
 
 # The single-layer configurations are instantiated with two layers: layer 0 is the
 # full-recompute layer and layer 1 the selective layer under test.
@@ -131,6 +150,9 @@ WORKLOADS: Dict[str, Workload] = {
     "tiny_sep": Workload("tiny-2L-4x126+sep2+32", TINY, 4, 126, 32, n_sep=2),
     "l8b_1layer_sep": Workload("llama8b-2L-8x478+sep2+64", LLAMA8B.with_layers(2), 8, 478, 64, n_sep=2),
     "l8b_124k_sep": Workload("llama8b-32L-242x512+sep2+128", LLAMA8B, 242, 512, 128, n_sep=2),
+    # YaRN RoPE, seven q heads per kv head, q/k/v bias
+    "yarn_tiny": Workload("yarn-gqa7-tiny-2L-4x128+32", YARN_GQA7_TINY, 4, 128, 32),
+    "yarn_2l": Workload("yarn-gqa7-2L-8x480+64", YARN_GQA7, 8, 480, 64),
 }
 
 
@@ -159,7 +181,8 @@ LAYER_TENSORS = ("w_qkv", "w_o", "w_gate", "w_up", "w_down")
 
 def make_layer_weights(shape: ModelShape, layer: int, seed: int = 0,
                        device: str | torch.device = "cpu") -> Dict[str, torch.Tensor]:
-    """One decoder layer: bf16 matrices (out_features x in_features) and fp32 gains.
+    """One decoder layer: bf16 matrices (out_features x in_features), fp32 gains and,
+    for shapes with one, the fp32 q/k/v bias `b_qkv` [qkv_dim].
 
     w_qkv rows are [q heads | k heads | v heads], each head `head_dim` rows.
     """
@@ -172,6 +195,8 @@ def make_layer_weights(shape: ModelShape, layer: int, seed: int = 0,
         "w_down": (H, F),
     }
     w = {n: randn_bf16(dims[n], tensor_seed(seed, layer, n), 0.02, device) for n in LAYER_TENSORS}
+    if shape.qkv_bias:
+        w["b_qkv"] = randn_bf16((shape.qkv_dim,), tensor_seed(seed, layer, "b_qkv"), 0.5, device).float()
     w["attn_norm"] = torch.ones(H, dtype=torch.float32, device=device)
     w["mlp_norm"] = torch.ones(H, dtype=torch.float32, device=device)
     return w

@@ -20,8 +20,12 @@ GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
 MINI = synth.ModelShape(hidden=64, n_q_heads=4, n_kv_heads=2, head_dim=16, mlp_dim=96,
                         n_layers=2, vocab=97, rms_eps=1e-5, rope_theta=10000.0)
+# seven q heads per kv head, YaRN (factor 4 over an original context of 16 tokens), q/k/v bias
+MINI_YARN = synth.ModelShape(hidden=64, n_q_heads=7, n_kv_heads=1, head_dim=16, mlp_dim=96,
+                             n_layers=2, vocab=97, rms_eps=1e-6, rope_theta=10000.0, rope_scaling=2,
+                             rs_factor=4.0, rs_low=1.0, rs_high=32.0, rs_orig_ctx=16, qkv_bias=True)
 MINI_L3 = synth.ModelShape(hidden=64, n_q_heads=4, n_kv_heads=2, head_dim=16, mlp_dim=96,
-                           n_layers=2, vocab=97, rms_eps=1e-5, rope_theta=500000.0, rope_llama3=True,
+                           n_layers=2, vocab=97, rms_eps=1e-5, rope_theta=500000.0, rope_scaling=1,
                            rs_factor=8.0, rs_low=1.0, rs_high=4.0, rs_orig_ctx=64)
 
 
@@ -93,8 +97,8 @@ def test_llama3_frequency_bands():
     """D=128, theta=5e5, orig 8192, low 1, high 4: wavelength 2*pi*theta^(2i/D) is below
     2048 for i <= 28 (kept), above 8192 for i >= 35 (divided by 8), and blended in between,
     continuously at both band edges."""
-    s = Shape(4096, 32, 8, 128, 14336, 1e-5, 500000.0, True, 8.0, 1.0, 4.0, 8192)
-    plain = Shape(4096, 32, 8, 128, 14336, 1e-5, 500000.0, False)
+    s = Shape(4096, 32, 8, 128, 14336, 1e-5, 500000.0, llama.ROPE_LLAMA3, 8.0, 1.0, 4.0, 8192)
+    plain = Shape(4096, 32, 8, 128, 14336, 1e-5, 500000.0, llama.ROPE_PLAIN)
     w = llama.rope_inv_freq(s)
     w0 = llama.rope_inv_freq(plain)
     assert w0[0] == 1.0 and abs(w0[1] - 500000.0 ** (-2 / 128)) < 1e-18
@@ -106,6 +110,102 @@ def test_llama3_frequency_bands():
     lam = 2 * math.pi / w0[mid]
     sm = (8192 / lam - 1.0) / 3.0
     assert np.all((sm > 0) & (sm < 1)) and np.all(np.diff(sm) < 0)
+
+
+def _yarn(D=128, theta=1e6, L=2048, scale=4.0, alpha=1.0, beta=32.0):
+    return Shape(4096, 32, 8, D, 14336, 1e-6, theta, llama.ROPE_YARN, scale, alpha, beta, L)
+
+
+def test_yarn_at_scale_one_is_plain_rope():
+    """s = 1: interpolation and extrapolation coincide, and the temperature is 1 (ln 1 = 0)."""
+    for D, theta, L in ((128, 1e6, 2048), (64, 1e4, 256)):
+        y = _yarn(D, theta, L, scale=1.0)
+        plain = Shape(4096, 32, 8, D, 14336, 1e-6, theta, llama.ROPE_PLAIN)
+        assert np.allclose(llama.rope_inv_freq(y), llama.rope_inv_freq(plain), rtol=1e-15, atol=0)
+        assert llama.logit_scale(y) == llama.logit_scale(plain) == 1.0 / math.sqrt(D)
+
+
+def test_yarn_bands_interpolate_and_keep():
+    """Pairs that turn fewer than alpha times over the original context L are position-
+    interpolated: their angle at position s*p equals the plain angle at p.  Pairs that
+    turn more than beta times keep the plain angle.  In between the frequency lies
+    strictly between the two and falls monotonically with the pair index."""
+    y = _yarn()
+    plain = Shape(4096, 32, 8, 128, 14336, 1e-6, 1e6, llama.ROPE_PLAIN)
+    w0 = llama.rope_inv_freq(plain)
+    turns = 2048 * w0 / (2 * math.pi)
+    low, high, mid = turns < 1.0, turns > 32.0, (turns >= 1.0) & (turns <= 32.0)
+    assert low.sum() > 10 and high.sum() > 5 and mid.sum() > 5
+    p = np.array([0, 1, 3, 1000, 30000])
+    cy, sy = llama.rope_cos_sin(y, 4 * p)
+    c0, s0 = llama.rope_cos_sin(plain, p)
+    assert np.allclose(cy[:, low], c0[:, low], atol=1e-9) and np.allclose(sy[:, low], s0[:, low], atol=1e-9)
+    cy, sy = llama.rope_cos_sin(y, p)
+    assert np.allclose(cy[:, high], c0[:, high], atol=1e-9) and np.allclose(sy[:, high], s0[:, high], atol=1e-9)
+    w = llama.rope_inv_freq(y)
+    assert np.all(w[mid] < w0[mid]) and np.all(w[mid] > w0[mid] / 4.0)
+    assert np.all(np.diff(w) < 0)
+
+
+def test_yarn_ramp_is_continuous_in_the_original_context():
+    """gamma is continuous, so a pair's frequency moves continuously as L crosses the
+    lengths at which it makes exactly alpha or beta turns."""
+    plain = Shape(4096, 32, 8, 128, 14336, 1e-6, 1e6, llama.ROPE_PLAIN)
+    w0 = llama.rope_inv_freq(plain)
+    d = 40
+    for n_turns in (1.0, 32.0):
+        L_edge = n_turns * 2 * math.pi / w0[d]
+        lo = llama.yarn_inv_freq(_yarn(L=L_edge * (1 - 1e-9)))[d]
+        hi = llama.yarn_inv_freq(_yarn(L=L_edge * (1 + 1e-9)))[d]
+        assert abs(lo - hi) < 1e-7 * w0[d]
+
+
+def test_yarn_equals_llama3_rule_with_the_same_bounds():
+    """Llama 3.1's frequency rule is the same NTK-by-parts blend (low/high frequency
+    factors in the roles of alpha/beta), written here independently: with equal
+    bounds the two definitions give the same frequencies."""
+    for D, theta, L, s_, a, b in ((128, 5e5, 8192, 8.0, 1.0, 4.0), (64, 1e4, 300, 3.0, 2.0, 16.0)):
+        y = _yarn(D, theta, L, s_, a, b)
+        l3 = Shape(4096, 32, 8, D, 14336, 1e-6, theta, llama.ROPE_LLAMA3, s_, a, b, L)
+        assert np.allclose(llama.rope_inv_freq(y), llama.rope_inv_freq(l3), rtol=1e-14, atol=0)
+
+
+def test_yarn_temperature_closed_form():
+    """Two keys, values 1 and 0: the output is the softmax weight of the first key,
+    sigmoid(c * (q.k1 - q.k2)).  With s = e^10, sqrt(1/t) = 0.1*10 + 1 = 2, so
+    c = 4/sqrt(D)."""
+    D = 16
+    y = Shape(64, 2, 1, D, 96, 1e-6, 1e4, llama.ROPE_YARN, math.exp(10.0), 1.0, 32.0, 64)
+    rng = np.random.default_rng(7)
+    q = rng.standard_normal((1, 2, D))
+    k = rng.standard_normal((2, 1, D))
+    v = np.zeros((2, 1, D)); v[0, 0, :] = 1.0
+    out = llama.attention_rows(y, q, k, v, [1])
+    for j in range(2):
+        delta = float(q[0, j] @ k[0, 0] - q[0, j] @ k[1, 0])
+        expect = 1.0 / (1.0 + math.exp(-4.0 * delta / math.sqrt(D)))
+        assert np.allclose(out[0, j], expect, rtol=1e-13)
+
+
+def test_qkv_bias_closed_form():
+    """Zero projection weights: q, k are the rotated bias and v the bias itself; the
+    key-only path adds the key slice of the same bias."""
+    s = Shape.of(MINI_YARN)
+    D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
+    rng = np.random.default_rng(8)
+    b = rng.standard_normal((Hq + 2 * Hkv) * D)
+    lw = {"attn_norm": np.ones(64), "w_qkv": np.zeros(((Hq + 2 * Hkv) * D, 64)), "b_qkv": b}
+    x = rng.standard_normal((3, 64))
+    pos = np.array([0, 5, 40])
+    q, k, v = llama.qkv_rows(s, lw, x, pos)
+    c, sn = llama.rope_cos_sin(s, pos)
+    assert np.allclose(q, llama.apply_rope(np.broadcast_to(b[: Hq * D].reshape(1, Hq, D), (3, Hq, D)), c, sn))
+    kb = b[Hq * D: (Hq + Hkv) * D].reshape(1, Hkv, D)
+    assert np.allclose(k, llama.apply_rope(np.broadcast_to(kb, (3, Hkv, D)), c, sn))
+    assert np.allclose(v, np.broadcast_to(b[(Hq + Hkv) * D:].reshape(1, Hkv, D), (3, Hkv, D)))
+    lw["w_qkv"] = rng.standard_normal(lw["w_qkv"].shape) * 0.1
+    q, k, v = llama.qkv_rows(s, lw, x, pos)
+    assert rel(llama.k_rows(s, lw, x, pos), k) < 1e-14
 
 
 # ------------------------------------------------------------------------------------ block parts
@@ -198,6 +298,31 @@ def test_layer_llama3_scaled_block_diagonal_matches_torch():
     inv = torch.as_tensor(llama.rope_inv_freq(s))
     ref, _, _ = torch_ref.layer_full(s, m["layers_np"][1], torch.as_tensor(x), inv, torch.as_tensor(pos), mask)
     assert rel(ours, ref.numpy()) < 1e-12
+
+
+def test_layer_yarn_gqa7_bias_matches_torch():
+    """Seven q heads per kv head, YaRN frequencies and temperature, q/k/v bias: the oracle's
+    layer against torch's block with the bias in F.linear and the temperature as SDPA's
+    scale, over positions up to 4x the original context."""
+    m = model(MINI_YARN)
+    s = Shape.of(MINI_YARN)
+    n = 64
+    x = llama.as64(synth.randn_bf16((n, 64), 13))
+    lw = m["layers_np"][0]
+    assert "b_qkv" in lw
+    kc = np.zeros((n, 1, 16)); vc = np.zeros_like(kc)
+    ours = llama.layer_rows(s, lw, x, np.arange(n), np.arange(n), kc, vc)
+    inv = torch.as_tensor(llama.rope_inv_freq(s))
+    mult = (0.1 * math.log(4.0) + 1.0) ** 2
+    ref, kr, vr = torch_ref.layer_full(s, lw, torch.as_tensor(x), inv, torch.arange(n), scale=mult / 4.0)
+    assert rel(ours, ref.numpy()) < 1e-12
+    assert rel(kc, kr.numpy()) < 1e-12 and rel(vc, vr.numpy()) < 1e-12
+    # without the temperature or the bias the layer differs
+    ref2, _, _ = torch_ref.layer_full(s, lw, torch.as_tensor(x), inv, torch.arange(n))
+    assert rel(ours, ref2.numpy()) > 1e-4
+    lw_nb = dict(lw); lw_nb.pop("b_qkv")
+    ref3, _, _ = torch_ref.layer_full(s, lw_nb, torch.as_tensor(x), inv, torch.arange(n), scale=mult / 4.0)
+    assert rel(ours, ref3.numpy()) > 1e-4
 
 
 # ------------------------------------------------------------------------------------ the method
@@ -347,10 +472,12 @@ def _pins_fail(monkeypatch, target, attr, bad):
     for t in (test_layer_matches_torch_library_block, test_attention_matches_sdpa_causal_gqa,
               test_rope_direction_closed_form, test_full_ratio_equals_full_prefill,
               test_prefix_invariance_and_realign, test_rope_matches_complex_multiplication,
-              test_llama3_frequency_bands):
+              test_llama3_frequency_bands, test_yarn_bands_interpolate_and_keep,
+              test_yarn_equals_llama3_rule_with_the_same_bounds, test_yarn_temperature_closed_form,
+              test_layer_yarn_gqa7_bias_matches_torch, test_qkv_bias_closed_form):
         try:
             t()
-        except AssertionError:
+        except (AssertionError, ValueError):   # a wrong result, or operands that no longer fit
             failed.append(t.__name__)
     monkeypatch.undo()
     return failed
@@ -387,6 +514,30 @@ def test_planted_mistakes(monkeypatch):
     def freq_bad(s):                   # exponent -i/D instead of -2i/D
         return good_freq(s) ** 0.5
     assert _pins_fail(monkeypatch, llama, "rope_inv_freq", freq_bad)
+
+    good_yarn = llama.yarn_inv_freq
+    def yarn_swapped(s):               # interpolation on the fast pairs instead of the slow ones
+        w = good_yarn(s)
+        plain = s.rope_theta ** (-2.0 * np.arange(s.head_dim // 2) / s.head_dim)
+        return plain * plain / w
+    assert _pins_fail(monkeypatch, llama, "yarn_inv_freq", yarn_swapped)
+
+    good_scale = llama.logit_scale
+    def temp_once(s):                  # temperature applied as sqrt(1/t) instead of 1/t
+        m = 0.1 * math.log(s.rs_factor) + 1.0 if s.rope_scaling == llama.ROPE_YARN else 1.0
+        return good_scale(s) / m
+    assert _pins_fail(monkeypatch, llama, "logit_scale", temp_once)
+
+    good_qkv = llama.qkv_rows
+    def qkv_bias_after_rope(s, lw, x, pos):   # bias added after the rotation
+        if lw.get("b_qkv") is None:
+            return good_qkv(s, lw, x, pos)
+        lw2 = dict(lw); b = llama.as64(lw2.pop("b_qkv"))
+        q, k, v = good_qkv(s, lw2, x, pos)
+        D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
+        return (q + b[: Hq * D].reshape(1, Hq, D), k + b[Hq * D:(Hq + Hkv) * D].reshape(1, Hkv, D),
+                v + b[(Hq + Hkv) * D:].reshape(1, Hkv, D))
+    assert _pins_fail(monkeypatch, llama, "qkv_rows", qkv_bias_after_rope)
 
 
 # ------------------------------------------------------------------------------------ bf16 storage mode

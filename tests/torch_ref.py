@@ -30,12 +30,15 @@ def rope_complex(x: torch.Tensor, pos: torch.Tensor, inv_freq: torch.Tensor) -> 
 
 
 def layer_full(s, lw: dict, x: torch.Tensor, inv_freq: torch.Tensor, pos: torch.Tensor,
-               attn_mask: torch.Tensor | None = None):
-    """Full layer over all n rows; attn_mask [n, n] boolean (True = may attend) or causal."""
+               attn_mask: torch.Tensor | None = None, scale: float | None = None):
+    """Full layer over all n rows; attn_mask [n, n] boolean (True = may attend) or causal.
+    The q/k/v projection takes lw["b_qkv"] as its bias when present; `scale` is the
+    softmax's logit factor (None: the library's default 1/sqrt(D))."""
     n = x.shape[0]
     D, Hq, Hkv = s.head_dim, s.n_q_heads, s.n_kv_heads
     n1 = F.rms_norm(x, (x.shape[-1],), weight=t64(lw["attn_norm"]), eps=s.rms_eps)
-    qkv = F.linear(n1, t64(lw["w_qkv"]))
+    b = lw.get("b_qkv")
+    qkv = F.linear(n1, t64(lw["w_qkv"]), None if b is None else t64(b))
     q = qkv[:, : Hq * D].reshape(n, Hq, D)
     k = qkv[:, Hq * D: (Hq + Hkv) * D].reshape(n, Hkv, D)
     v = qkv[:, (Hq + Hkv) * D:].reshape(n, Hkv, D)
@@ -46,9 +49,9 @@ def layer_full(s, lw: dict, x: torch.Tensor, inv_freq: torch.Tensor, pos: torch.
     vv = v.repeat_interleave(grp, dim=1)
     qh, kh, vh = (t.transpose(0, 1)[None] for t in (q, kk, vv))
     if attn_mask is None:
-        o = F.scaled_dot_product_attention(qh, kh, vh, is_causal=True)
+        o = F.scaled_dot_product_attention(qh, kh, vh, is_causal=True, scale=scale)
     else:
-        o = F.scaled_dot_product_attention(qh, kh, vh, attn_mask=attn_mask[None, None])
+        o = F.scaled_dot_product_attention(qh, kh, vh, attn_mask=attn_mask[None, None], scale=scale)
     o = o[0].transpose(0, 1).reshape(n, Hq * D)
     h = x + F.linear(o, t64(lw["w_o"]))
     n2 = F.rms_norm(h, (h.shape[-1],), weight=t64(lw["mlp_norm"]), eps=s.rms_eps)
