@@ -60,14 +60,26 @@ typedef enum kvb_status {
     KVB_ERR_WORKSPACE = 5      /* workspace missing or smaller than required            */
 } kvb_status;
 
-/* Model shape and RoPE settings (Llama 3.1 frequency scaling when rope_llama3 != 0:
- * factor rs_factor, low/high frequency factors rs_low/rs_high, original context
- * rs_orig_ctx). */
+/* Frequency scaling of the rotary embedding (kvb_config.rope_scaling). */
+enum {
+    KVB_ROPE_PLAIN = 0,    /* w_i = theta^(-2i/D)                                            */
+    KVB_ROPE_LLAMA3 = 1,   /* Llama 3.1: factor rs_factor, low/high frequency factors
+                            * rs_low/rs_high, original context rs_orig_ctx                   */
+    KVB_ROPE_YARN = 2      /* YaRN (the scaling of the paper's second model, Sec. 4): NTK-by-
+                            * parts interpolation with scale s = rs_factor >= 1, ramp bounds
+                            * alpha = rs_low < beta = rs_high (turns of a pair over the
+                            * original context rs_orig_ctx), and the attention logits
+                            * multiplied by (0.1 ln s + 1)^2 (YaRN's temperature)            */
+};
+
+/* Model shape and RoPE settings.  Hq must be a multiple of Hkv; any group size
+ * Hq/Hkv <= 128 runs in the prefill, the decode attention is built for group sizes
+ * 1, 2, 4, 7 and 8. */
 typedef struct kvb_config {
     int32_t hidden, n_q_heads, n_kv_heads, head_dim, mlp_dim, n_layers, vocab;
     float rms_eps;
     float rope_theta;
-    int32_t rope_llama3;
+    int32_t rope_scaling;                 /* KVB_ROPE_*                               */
     float rs_factor, rs_low, rs_high;
     int32_t rs_orig_ctx;
 } kvb_config;
@@ -83,6 +95,8 @@ typedef struct kvb_layer_weights {
     const uint16_t* w_gate;
     const uint16_t* w_up;
     const uint16_t* w_down;
+    const float* b_qkv;   /* fp32 [(Hq+2Hkv)D] bias of the q/k/v projection (added before
+                           * RoPE), or NULL for none                                      */
 } kvb_layer_weights;
 
 /* Whole model: `layers` is a HOST array of n_layers entries; embed is [vocab][H] bf16,
@@ -140,12 +154,20 @@ int32_t kvb_version(void);
 /* ------------------------------------------------------------------ RoPE */
 
 /* Fill HOST tables cos_host/sin_host, each [max_pos][D/2] fp32, with cos/sin of
- * pos * w_i for pos < max_pos (w_i = theta^(-2i/D), Llama 3.1 scaling if enabled;
+ * pos * w_i for pos < max_pos (w_i = theta^(-2i/D) under cfg->rope_scaling;
  * Sec. 4 asks for the position adjustment in float32 - angles are formed in double
- * and rounded once).  Pure host call.  Errors: INVALID_ARG for NULL pointers,
- * max_pos < 1 or an unsupported head_dim. */
+ * and rounded once).  The tables hold pure rotations: YaRN's temperature is applied
+ * to the attention logits (kvb_attention_scale), not folded into cos/sin, so that the
+ * re-alignment of cached keys stays a rotation.  Pure host call.  Errors: INVALID_ARG
+ * for NULL pointers, max_pos < 1, an unknown scaling or bad scaling parameters,
+ * UNSUPPORTED for a head_dim that is not built. */
 kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos,
                                float* cos_host, float* sin_host);
+
+/* The factor every attention kernel applies to q.k before the softmax: 1/sqrt(D),
+ * times (0.1 ln s + 1)^2 under KVB_ROPE_YARN (YaRN, Sec. 3.4 of its paper).  Pure
+ * host call.  Errors: INVALID_ARG for NULL pointers or an invalid config. */
+kvb_status kvb_attention_scale(const kvb_config* cfg, float* scale_out);
 
 /* ------------------------------------------------------------------ steps */
 

@@ -148,12 +148,35 @@ static kvb_status check_cfg(const kvb_config* c) {
         return fail(KVB_ERR_INVALID_ARG, "config: sizes must be positive");
     if (c->head_dim != 64 && c->head_dim != 128)
         return fail(KVB_ERR_UNSUPPORTED, "config: head_dim %d not built (64 or 128)", c->head_dim);
-    if (c->n_q_heads % c->n_kv_heads || 128 % (c->n_q_heads / c->n_kv_heads))
-        return fail(KVB_ERR_UNSUPPORTED, "config: Hq/Hkv must divide 128");
-    if (c->hidden % 256) return fail(KVB_ERR_UNSUPPORTED, "config: hidden must be a multiple of 256");
+    if (c->n_q_heads % c->n_kv_heads || c->n_q_heads / c->n_kv_heads > 128)
+        return fail(KVB_ERR_UNSUPPORTED, "config: Hq must be a multiple of Hkv with Hq/Hkv <= 128");
+    if (c->hidden % 256 || c->hidden > 8192)
+        return fail(KVB_ERR_UNSUPPORTED, "config: hidden must be a multiple of 256, at most 8192");
     if (c->mlp_dim % 16) return fail(KVB_ERR_UNSUPPORTED, "config: mlp_dim must be a multiple of 16");
     if (!(c->rms_eps >= 0.f) || !(c->rope_theta > 0.f)) return fail(KVB_ERR_INVALID_ARG, "config: eps/theta");
+    if (c->rope_scaling != KVB_ROPE_PLAIN && c->rope_scaling != KVB_ROPE_LLAMA3 && c->rope_scaling != KVB_ROPE_YARN)
+        return fail(KVB_ERR_INVALID_ARG, "config: unknown rope_scaling %d", c->rope_scaling);
+    if (c->rope_scaling != KVB_ROPE_PLAIN) {
+        const float min_factor = c->rope_scaling == KVB_ROPE_YARN ? 1.f : 0.f;
+        if (!(c->rs_factor >= min_factor) || !(c->rs_factor > 0.f) || !(c->rs_low > 0.f) ||
+            !(c->rs_high > c->rs_low) || c->rs_orig_ctx < 1)
+            return fail(KVB_ERR_INVALID_ARG, "config: rope scaling needs factor > 0 (>= 1 for YaRN), "
+                        "0 < low < high and an original context >= 1");
+    }
     return KVB_OK;
+}
+
+// q.k multiplier of the softmax, times log2(e) (the kernels exponentiate base 2)
+static double attn_scale(const kvb_config* c) {
+    double s = 1.0 / sqrt((double)c->head_dim);
+    if (c->rope_scaling == KVB_ROPE_YARN) {
+        const double m = 0.1 * log((double)c->rs_factor) + 1.0;   // YaRN: sqrt(1/t)
+        s *= m * m;
+    }
+    return s;
+}
+static float attn_scale_log2(const kvb_config* c) {
+    return (float)(1.4426950408889634 * attn_scale(c));
 }
 
 static kvb_status check_ptr(const void* p, const char* name) {
@@ -170,6 +193,7 @@ static kvb_status check_layer(const kvb_layer_weights* w) {
         (s = check_ptr(w->w_gate, "w_gate")) || (s = check_ptr(w->w_up, "w_up")) ||
         (s = check_ptr(w->w_down, "w_down")))
         return s;
+    if (w->b_qkv && !aligned16(w->b_qkv)) return fail(KVB_ERR_INVALID_ARG, "b_qkv is not 16-byte aligned");
     return KVB_OK;
 }
 
@@ -189,19 +213,30 @@ static kvb_status check_rope(const kvb_rope_table* r, int64_t need_pos) {
         if (_s != KVB_OK) return _s;     \
     } while (0)
 
+// Rotation frequency of every pair i < D/2 under the config's scaling.
 static void inv_freq(const kvb_config* c, double* w) {
     const int D = c->head_dim;
+    const double two_pi = 2.0 * 3.14159265358979323846;
     for (int i = 0; i < D / 2; ++i) {
         const double f = pow((double)c->rope_theta, -(2.0 * i) / D);
-        if (!c->rope_llama3) { w[i] = f; continue; }
-        const double lam = 2.0 * 3.14159265358979323846 / f;
-        const double hi_wl = c->rs_orig_ctx / (double)c->rs_high;   // shortest blended wavelength
-        const double lo_wl = c->rs_orig_ctx / (double)c->rs_low;    // longest blended wavelength
-        if (lam < hi_wl) w[i] = f;
-        else if (lam > lo_wl) w[i] = f / c->rs_factor;
-        else {
-            const double s = (c->rs_orig_ctx / lam - c->rs_low) / ((double)c->rs_high - c->rs_low);
-            w[i] = (1.0 - s) * f / c->rs_factor + s * f;
+        if (c->rope_scaling == KVB_ROPE_PLAIN) { w[i] = f; continue; }
+        const double lam = two_pi / f;   // wavelength in tokens
+        if (c->rope_scaling == KVB_ROPE_LLAMA3) {
+            const double hi_wl = c->rs_orig_ctx / (double)c->rs_high;   // shortest blended wavelength
+            const double lo_wl = c->rs_orig_ctx / (double)c->rs_low;    // longest blended wavelength
+            if (lam < hi_wl) w[i] = f;
+            else if (lam > lo_wl) w[i] = f / c->rs_factor;
+            else {
+                const double s = (c->rs_orig_ctx / lam - c->rs_low) / ((double)c->rs_high - c->rs_low);
+                w[i] = (1.0 - s) * f / c->rs_factor + s * f;
+            }
+        } else {
+            // YaRN NTK-by-parts: r = turns of the pair over the original context; ramp
+            // gamma(r) from interpolation (f / s, below alpha turns) to f (above beta)
+            const double r = c->rs_orig_ctx / lam;
+            const double a = c->rs_low, b = c->rs_high;
+            const double gamma = r < a ? 0.0 : (r > b ? 1.0 : (r - a) / (b - a));
+            w[i] = (1.0 - gamma) * f / c->rs_factor + gamma * f;
         }
     }
 }
@@ -275,7 +310,7 @@ kvb_status qkv_rows(const Ctx& x, const kvb_layer_weights* lw, const float* xin,
     p.M = m; p.N = x.QD + 2 * x.KVD; p.K = x.H; p.epi = EPI_QKV;
     p.col_base = 0; p.q_dim = x.QD; p.kv_dim = x.KVD; p.head_dim = x.D;
     p.q_out = q; p.k_out = k; p.v_out = v; p.kv_dst = kv_dst; p.rope_pos = rope_pos;
-    p.cos_t = x.rope->cos; p.sin_t = x.rope->sin; p.status = x.w.status;
+    p.cos_t = x.rope->cos; p.sin_t = x.rope->sin; p.bias = lw->b_qkv; p.status = x.w.status;
     return gemm(x, p, x.w.a, x.H, lw->w_qkv, x.H, nullptr);
 }
 
@@ -298,7 +333,7 @@ kvb_status attn_rows(const Ctx& x, const uint16_t* q, const int32_t* q_idx, cons
     AttnParams a{};
     a.q_idx = q_idx; a.kv_lo = kv_lo; a.m = m; a.n_kv = n_kv;
     a.Hq = x.Hq; a.Hkv = x.Hkv; a.D = x.D; a.out = out;
-    a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)x.D));
+    a.scale_log2 = attn_scale_log2(x.c);
     a.status = x.w.status;
     const int i = x.prof ? x.prof->begin(selective ? PK_ATTN_SEL : PK_ATTN_DENSE) : -1;
     kvb_status s = launch_attn(a, q, kc, vc, x.st);
@@ -374,7 +409,7 @@ const char* kvb_status_string(kvb_status s) {
 
 const char* kvb_last_error(void) { return g_err; }
 
-int32_t kvb_version(void) { return 100; }
+int32_t kvb_version(void) { return 200; }
 
 kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos, float* cos_host, float* sin_host) {
     g_err[0] = 0;
@@ -389,6 +424,14 @@ kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos, float* co
             cos_host[p * half + i] = (float)cos(a);
             sin_host[p * half + i] = (float)sin(a);
         }
+    return KVB_OK;
+}
+
+kvb_status kvb_attention_scale(const kvb_config* cfg, float* scale_out) {
+    g_err[0] = 0;
+    KVB_TRY(check_cfg(cfg));
+    if (!scale_out) return fail(KVB_ERR_INVALID_ARG, "attention scale: NULL output");
+    *scale_out = (float)attn_scale(cfg);
     return KVB_OK;
 }
 
@@ -727,7 +770,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
                 p.M = n_ctx; p.N = c.KVD; p.K = c.H; p.epi = EPI_QKV;
                 p.col_base = c.QD; p.q_dim = c.QD; p.kv_dim = c.KVD; p.head_dim = c.D;
                 p.k_out = w.k_fresh; p.rope_pos = w.ident; p.cos_t = rope->cos; p.sin_t = rope->sin;
-                p.status = w.status;
+                p.bias = lw->b_qkv; p.status = w.status;
                 KVB_TRY(gemm(c, p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr));
                 KVB_TRY(wait_layer(lc));
                 const int hp = c.prof ? c.prof->begin(PK_HKVD) : -1;
@@ -918,6 +961,9 @@ static kvb_status check_decode(const kvb_config* cfg, int64_t max_pos) {
     const int64_t qd = (int64_t)cfg->n_q_heads * cfg->head_dim;
     if (cfg->hidden > KVB_DECODE_MAX_K || cfg->mlp_dim > KVB_DECODE_MAX_K || qd > KVB_DECODE_MAX_K)
         return fail(KVB_ERR_UNSUPPORTED, "decode: hidden, mlp_dim and Hq*D must be at most %d", KVB_DECODE_MAX_K);
+    const int G = cfg->n_q_heads / cfg->n_kv_heads;
+    if (G != 1 && G != 2 && G != 4 && G != 7 && G != 8)
+        return fail(KVB_ERR_UNSUPPORTED, "decode: %d q heads per kv head not built (1, 2, 4, 7, 8)", G);
     return KVB_OK;
 }
 
@@ -946,7 +992,7 @@ kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const 
     const size_t need = decode_layout(cfg, max_pos, nullptr, &w);
     if (!ws || ws_bytes < need) return fail(KVB_ERR_WORKSPACE, "decode attention: workspace %zu < %zu", ws_bytes, need);
     decode_layout(cfg, max_pos, ws, &w);
-    const float sl2 = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
+    const float sl2 = attn_scale_log2(cfg);
     return launch_decode_attn(q, k_layer, v_layer, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, pos, max_pos, sl2,
                               w.pm, w.pl, w.po, out, w.status, static_cast<cudaStream_t>(stream));
 }
@@ -972,7 +1018,7 @@ kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const 
     const int H = cfg->hidden, F = cfg->mlp_dim, D = cfg->head_dim, Hq = cfg->n_q_heads, Hkv = cfg->n_kv_heads;
     const int QD = Hq * D, KVD = Hkv * D;
     const float eps = cfg->rms_eps;
-    const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));
+    const float sl2 = attn_scale_log2(cfg);
     float* hidden = hidden_out ? hidden_out : w.hidden;
     KVB_TRY(launch_decode_embed(model->embed, tokens, pos, max_pos, cfg->vocab, H, w.x, w.status, st));
     GemvArgs ga{};
@@ -988,7 +1034,7 @@ kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const 
         uint16_t* kc = cache->k + (int64_t)l * cache->n_rows * KVD;
         uint16_t* vc = cache->v + (int64_t)l * cache->n_rows * KVD;
         GemvArgs qkv = ga;                     // RMSNorm + QKV + RoPE + K/V append
-        qkv.W = lw.w_qkv; qkv.K = H; qkv.x = w.x; qkv.g = lw.attn_norm;
+        qkv.W = lw.w_qkv; qkv.bias = lw.b_qkv; qkv.K = H; qkv.x = w.x; qkv.g = lw.attn_norm;
         qkv.q_out = w.q; qkv.k_layer = kc; qkv.v_layer = vc;
         KVB_TRY(launch_gemv(GEMV_QKV, qkv, st));
         KVB_TRY(launch_decode_attn(w.q, kc, vc, Hq, Hkv, D, pos, max_pos, sl2, w.pm, w.pl, w.po, w.attn, w.status, st));

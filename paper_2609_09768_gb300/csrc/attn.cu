@@ -1,9 +1,9 @@
 // Sparse-query causal GQA flash attention on the 5th-generation tensor cores.
 //
-// Each CTA owns one (block of query rows, kv head) unit.  The Hq/Hkv query heads
-// that share kv head g are packed with 128/(Hq/Hkv) query rows into the 128 rows
-// of one MMA tile (lane = row_in_block * G + head_in_group), so every K/V tile
-// loaded serves all G heads.  Row r attends cache rows [lo_r, hi_r] where hi_r is
+// Each CTA owns one (block of query rows, kv head) unit.  The G = Hq/Hkv query heads
+// that share kv head g are packed with RPB = floor(128/G) query rows into the 128
+// rows of one MMA tile (lane = row_in_block * G + head_in_group; the last 128 - RPB*G
+// lanes idle when G does not divide 128), so every K/V tile loaded serves all G heads.  Row r attends cache rows [lo_r, hi_r] where hi_r is
 // the row's own cache index: this one predicate covers the sparse recompute rows
 // of the selective layers, the dense causal prefill and the block-diagonal
 // per-chunk prefill.
@@ -106,7 +106,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     const int L = (int)(quarter * 32 + lane);
     const int64_t row = r0 + L / G;
     const int head = g * G + L % G;
-    const bool valid = warp >= 2 && row < p.m;
+    const bool valid = warp >= 2 && L < RPB * G && row < p.m;
     int hi = -1, lo = 0;
     if (valid) {
         hi = p.q_idx[row];
@@ -359,8 +359,8 @@ kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k
                        cudaStream_t st) {
     if (p.m <= 0) return KVB_OK;
     if (p.D != 64 && p.D != 128) return fail(KVB_ERR_UNSUPPORTED, "attention: head_dim %d not built", p.D);
-    if (p.Hkv <= 0 || p.Hq % p.Hkv || 128 % (p.Hq / p.Hkv))
-        return fail(KVB_ERR_UNSUPPORTED, "attention: Hq/Hkv must divide 128");
+    if (p.Hkv <= 0 || p.Hq % p.Hkv || p.Hq / p.Hkv > 128)
+        return fail(KVB_ERR_UNSUPPORTED, "attention: Hq must be a multiple of Hkv with Hq/Hkv <= 128");
     const int G = p.Hq / p.Hkv, RPB = 128 / G;
     CUtensorMap tk, tv;
     const uint64_t kvd = (uint64_t)p.Hkv * p.D;

@@ -14,8 +14,8 @@
 //                       up rows in one warp
 //   decode_attn       - split-KV attention of the new row over cache rows [0, pos]:
 //                       one warp per split of 128 keys and kv head, lanes over head
-//                       dims; the G q heads sharing the kv head and 32/G keys give 32
-//                       partial dot products per step, summed with one 31-shuffle
+//                       dims; the G q heads sharing the kv head (padded to a power of
+//                       two GP) and 32/GP keys give 32 partial dot products per step, summed with one 31-shuffle
 //                       reduce-scatter; online softmax per head in fp32; the next
 //                       step's K/V loads are issued before this step's arithmetic; the 8
 //                       warps of a CTA merge their (max, sum, O) in shared memory
@@ -111,8 +111,8 @@ KVB_DEV void dot_rows(const uint16_t* __restrict__ w1, const uint16_t* __restric
 //                          normalises it itself: no separate norm launch);
 //   GEMV_RESID:            the bf16 row `a` as given.
 // Work units per warp:
-//   GEMV_QKV    - a rotation pair (rows i and i + D/2 of a q or k head): RoPE at `pos`,
-//                 bf16 q or cache K row `pos`; or one V row: cache V row `pos`
+//   GEMV_QKV    - a rotation pair (rows i and i + D/2 of a q or k head): bias, RoPE at
+//                 `pos`, bf16 q or cache K row `pos`; or one V row (+ bias): cache V row `pos`
 //   GEMV_RESID  - one row: x[n] += y
 //   GEMV_SWIGLU - gate row n and up row n: h[n] = bf16(silu(gate) * up)
 template <int MODE>
@@ -164,6 +164,10 @@ gemv_kernel(const GemvArgs p) {
                 dot_rows<true, 8>(p.W + ((int64_t)h * D + i) * K, p.W + ((int64_t)h * D + i + half) * K, act, K, lane,
                                   a, b);
                 if (lane == 0) {
+                    if (p.bias) {
+                        a += p.bias[(int64_t)h * D + i];
+                        b += p.bias[(int64_t)h * D + i + half];
+                    }
                     const float c = p.cos_t[(int64_t)pos * half + i], sn = p.sin_t[(int64_t)pos * half + i];
                     const float y1 = a * c - b * sn;
                     const float y2 = b * c + a * sn;
@@ -176,6 +180,7 @@ gemv_kernel(const GemvArgs p) {
                 float a, unused;
                 dot_rows<false, 16>(p.W + ((int64_t)(Hq + Hkv) * D + j) * K, nullptr, act, K, lane, a, unused);
                 if (lane == 0) {
+                    if (p.bias) a += p.bias[(int64_t)(Hq + Hkv) * D + j];
                     const float v = __bfloat162float(__float2bfloat16_rn(a));
                     p.v_layer[(int64_t)pos * Hkv * D + j] = __half_as_ushort(__float2half_rn(v));
                 }
@@ -212,6 +217,11 @@ KVB_DEV RowBits<DPL> load_row(const uint16_t* p) {
     return r;
 }
 
+// Head slots per kv head: the lane layout pads a group of G q heads to GP slots, a power
+// of two and at least 4 (so that a step covers at most 8 keys and the K/V prefetch fits in
+// registers); the padding heads have q = 0 and are never written out.
+__host__ __device__ constexpr int pad_pow2(int g) { return g <= 4 ? 4 : 8; }
+
 // One CTA = eight consecutive splits of KVB_DECODE_KEYS_PER_SPLIT cache rows for kv head
 // blockIdx.y, one warp per split; the warps' partial results are merged in shared memory
 // and the CTA writes one partial (max, sum, O) per q head.
@@ -221,10 +231,12 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
                    int Hkv, const int32_t* __restrict__ pos_ptr, int64_t max_pos, int n_blocks, float scale_log2,
                    float* __restrict__ pm, float* __restrict__ pl, float* __restrict__ po, int* status) {
     constexpr int DPL = D / 32;      // head dims per lane
-    constexpr int KS = 32 / G;       // keys per step: KS * G = 32 partial dot products
+    constexpr int GP = pad_pow2(G);  // head slots
+    static_assert(G >= 1 && G <= 8, "group size");
+    constexpr int KS = 32 / GP;      // keys per step: KS * GP = 32 partial dot products
     constexpr int WARPS = ATT_THREADS / 32;
-    __shared__ float sm_m[WARPS][G], sm_l[WARPS][G];
-    __shared__ float sm_o[WARPS][G][D];
+    __shared__ float sm_m[WARPS][GP], sm_l[WARPS][GP];
+    __shared__ float sm_o[WARPS][GP][D];
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
     if ((int)blockIdx.x >= n_blocks) return;
@@ -235,18 +247,20 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
     int64_t end = start + KVB_DECODE_KEYS_PER_SPLIT;
     if (end > (int64_t)pos + 1) end = (int64_t)pos + 1;
 
-    // q of the G heads in shared memory (registers go to the K/V prefetch)
-    __shared__ __align__(16) float qs[G][D];
+    // q of the G heads (zero for the padding slots) in shared memory (registers go to the
+    // K/V prefetch)
+    __shared__ __align__(16) float qs[GP][D];
     __shared__ __align__(16) float sp[ATT_THREADS / 32][32];   // per warp: this step's weights
-    __shared__ float sa[ATT_THREADS / 32][G];                   // per warp: rescale factor per head
-    for (int i = threadIdx.x; i < G * D; i += ATT_THREADS) qs[i / D][i % D] = bf16_to_f(q[(g * G) * D + i]);
+    __shared__ float sa[ATT_THREADS / 32][GP];                  // per warp: rescale factor per head
+    for (int i = threadIdx.x; i < GP * D; i += ATT_THREADS)
+        qs[i / D][i % D] = i < G * D ? bf16_to_f(q[(g * G) * D + i]) : 0.f;
     __syncthreads();
-    float o[G][DPL];
+    float o[GP][DPL];
 #pragma unroll
-    for (int h = 0; h < G; ++h)
+    for (int h = 0; h < GP; ++h)
 #pragma unroll
         for (int e = 0; e < DPL; ++e) o[h][e] = 0.f;
-    float m_run = -INFINITY, l_run = 0.f;    // of head lane % G
+    float m_run = -INFINITY, l_run = 0.f;    // of head slot lane % GP
 
     const int64_t row_stride = (int64_t)Hkv * D;
     const uint16_t* kbase = kc + (int64_t)g * D + lane * DPL;
@@ -270,9 +284,9 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
         if (k0 + KS < end) fetch(k0 + KS, nk, nv);
         float sc[32];
         {
-            float qv[G][DPL];   // this lane's head dims of q, once per step
+            float qv[GP][DPL];   // this lane's head dims of q, once per step
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
+            for (int h = 0; h < GP; ++h) {
                 if constexpr (DPL == 4) {
                     const float4 t4 = *reinterpret_cast<const float4*>(&qs[h][lane * 4]);
                     qv[h][0] = t4.x; qv[h][1] = t4.y; qv[h][2] = t4.z; qv[h][3] = t4.w;
@@ -287,11 +301,11 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
 #pragma unroll
                 for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
 #pragma unroll
-                for (int h = 0; h < G; ++h) {
+                for (int h = 0; h < GP; ++h) {
                     float acc = 0.f;
 #pragma unroll
                     for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[e], acc);
-                    sc[k * G + h] = acc;
+                    sc[k * GP + h] = acc;
                 }
             }
         }
@@ -307,26 +321,26 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
             }
         }
         float t = sc[0] * scale_log2;
-        if (k0 + lane / G >= end) t = -INFINITY;
-        // online softmax of head lane % G over this step's keys
+        if (k0 + lane / GP >= end) t = -INFINITY;
+        // online softmax of head slot lane % GP over this step's keys
         float mx = t;
 #pragma unroll
-        for (int off = G; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        for (int off = GP; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
         const float m_new = fmaxf(m_run, mx);
         const float alpha = (m_new == -INFINITY) ? 1.f : fast_exp2(m_run - m_new);
         const float pv = (t == -INFINITY) ? 0.f : fast_exp2(t - m_new);
         float ps = pv;
 #pragma unroll
-        for (int off = G; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+        for (int off = GP; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
         l_run = l_run * alpha + ps;
         m_run = m_new;
-        // this step's weights (index key * G + head) and the heads' rescale factors to every lane
+        // this step's weights (index key * GP + head) and the heads' rescale factors to every lane
         __syncwarp();
         sp[warp][lane] = pv;
-        if (lane < G) sa[warp][lane] = alpha;
+        if (lane < GP) sa[warp][lane] = alpha;
         __syncwarp();
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
+        for (int h = 0; h < GP; ++h) {
             const float ah = sa[warp][h];
 #pragma unroll
             for (int e = 0; e < DPL; ++e) o[h][e] *= ah;
@@ -339,22 +353,21 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
                 const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&cv[k].w[i]));
                 vf[2 * i] = f.x; vf[2 * i + 1] = f.y;
             }
+            float pk[GP];   // weights of key k for the GP head slots, vector loads (broadcast)
+            if constexpr (GP % 4 == 0) {
 #pragma unroll
-            float pk[G];   // weights of key k for the G heads, vector loads (broadcast)
-            if constexpr (G % 4 == 0) {
-#pragma unroll
-                for (int h4 = 0; h4 < G; h4 += 4) {
-                    const float4 t = *reinterpret_cast<const float4*>(&sp[warp][k * G + h4]);
+                for (int h4 = 0; h4 < GP; h4 += 4) {
+                    const float4 t = *reinterpret_cast<const float4*>(&sp[warp][k * GP + h4]);
                     pk[h4] = t.x; pk[h4 + 1] = t.y; pk[h4 + 2] = t.z; pk[h4 + 3] = t.w;
                 }
+            } else if constexpr (GP == 2) {
+                const float2 t = *reinterpret_cast<const float2*>(&sp[warp][k * GP]);
+                pk[0] = t.x; pk[1] = t.y;
             } else {
-#pragma unroll
-                for (int h2 = 0; h2 < G; h2 += 2) {
-                    const float2 t = *reinterpret_cast<const float2*>(&sp[warp][k * G + h2]);
-                    pk[h2] = t.x; pk[h2 + 1] = t.y;
-                }
+                pk[0] = sp[warp][k];
             }
-            for (int h = 0; h < G; ++h) {
+#pragma unroll
+            for (int h = 0; h < GP; ++h) {
 #pragma unroll
                 for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk[h], vf[e], o[h][e]);
             }
@@ -362,7 +375,7 @@ decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ 
 #pragma unroll
         for (int k = 0; k < KS; ++k) { ck[k] = nk[k]; cv[k] = nv[k]; }
     }
-    // merge the warps of this CTA
+    // merge the warps of this CTA (the G real heads)
 #pragma unroll
     for (int h = 0; h < G; ++h)
 #pragma unroll
@@ -499,11 +512,12 @@ kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint1
     const int G = Hq / Hkv;
     const int n_splits = decode_splits(max_pos, Hkv);
     kvb_status s;
-    if (D == 128 && G == 4) s = run_attn<128, 4>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
-    else if (D == 128 && G == 8) s = run_attn<128, 8>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
-    else if (D == 128 && G == 2) s = run_attn<128, 2>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
-    else if (D == 64 && G == 2) s = run_attn<64, 2>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
-    else if (D == 64 && G == 4) s = run_attn<64, 4>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
+#define KVB_DECODE_CASE(DD, GG) \
+    else if (D == DD && G == GG) s = run_attn<DD, GG>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
+    if (false) {}
+    KVB_DECODE_CASE(128, 1) KVB_DECODE_CASE(128, 2) KVB_DECODE_CASE(128, 4) KVB_DECODE_CASE(128, 7) KVB_DECODE_CASE(128, 8)
+    KVB_DECODE_CASE(64, 1) KVB_DECODE_CASE(64, 2) KVB_DECODE_CASE(64, 4) KVB_DECODE_CASE(64, 7) KVB_DECODE_CASE(64, 8)
+#undef KVB_DECODE_CASE
     else return fail(KVB_ERR_UNSUPPORTED, "decode attention: head_dim %d with %d q heads per kv head not built", D, G);
     if (s != KVB_OK) return s;
     decode_combine_kernel<<<dim3((unsigned)Hq, (unsigned)(D / 32)), 32 * COMB_GROUPS, 0, st>>>(

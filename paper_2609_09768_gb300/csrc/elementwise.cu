@@ -98,7 +98,8 @@ embed_kernel(const uint16_t* __restrict__ embed, const int32_t* __restrict__ tok
 }
 
 // ------------------------------------------------------------------ RMSNorm
-// One CTA of T threads per row; every thread holds V float4 of the row.
+// One CTA of T threads per row; thread t holds float4 t, t + T, ... (at most V of them)
+// of the row's H/4 float4.
 template <int T, int V>
 __global__ void __launch_bounds__(T)
 rmsnorm_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int64_t m, int H,
@@ -107,11 +108,13 @@ rmsnorm_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int
     const int64_t r = blockIdx.x;
     const int64_t src = idx ? (int64_t)__ldg(idx + r) : r;
     const float4* xr = reinterpret_cast<const float4*>(x + src * H);
+    const int H4 = H / 4;
     float4 v[V];
     float ss = 0.f;
 #pragma unroll
     for (int i = 0; i < V; ++i) {
-        v[i] = xr[threadIdx.x + i * T];
+        const int c = threadIdx.x + i * T;
+        v[i] = c < H4 ? xr[c] : make_float4(0.f, 0.f, 0.f, 0.f);
         ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
     }
 #pragma unroll
@@ -126,6 +129,7 @@ rmsnorm_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int
 #pragma unroll
     for (int i = 0; i < V; ++i) {
         const int c = threadIdx.x + i * T;
+        if (c >= H4) break;
         const float4 gg = __ldg(gr + c);
         const float4 y = make_float4(v[i].x * inv * gg.x, v[i].y * inv * gg.y, v[i].z * inv * gg.z, v[i].w * inv * gg.w);
         if (out_bf16) {
@@ -218,18 +222,14 @@ kvb_status launch_rmsnorm(const float* x, const int32_t* idx, int64_t m, int H, 
     if (m <= 0) return KVB_OK;
     if (m > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "rmsnorm: too many rows");
     const unsigned grid = (unsigned)m;
-    switch (H) {
-        case 4096: rmsnorm_kernel<128, 8><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32); break;
-        case 2048: rmsnorm_kernel<128, 4><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32); break;
-        case 1024: rmsnorm_kernel<128, 2><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32); break;
-        case 512:  rmsnorm_kernel<128, 1><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32); break;
-        case 256:  rmsnorm_kernel<64, 1><<<grid, 64, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32); break;
-        default:
-            if (H % 512 == 0 && H <= 8192)
-                rmsnorm_kernel<128, 16><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
-            else
-                return fail(KVB_ERR_UNSUPPORTED, "rmsnorm: hidden %d not built", H);
-    }
+    // 128 threads, each holding at most V float4 of the row (64 threads for H = 256)
+    if (H <= 0 || H % 4 || H > 8192) return fail(KVB_ERR_UNSUPPORTED, "rmsnorm: hidden %d not built", H);
+    if (H == 256) rmsnorm_kernel<64, 1><<<grid, 64, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
+    else if (H <= 512) rmsnorm_kernel<128, 1><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
+    else if (H <= 1024) rmsnorm_kernel<128, 2><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
+    else if (H <= 2048) rmsnorm_kernel<128, 4><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
+    else if (H <= 4096) rmsnorm_kernel<128, 8><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
+    else rmsnorm_kernel<128, 16><<<grid, 128, 0, st>>>(x, idx, m, H, g, eps, out_bf16, out_f32);
     count_launch();
     return cuda_ok(cudaGetLastError(), "rmsnorm launch");
 }

@@ -1,6 +1,6 @@
 // Row GEMM on the 5th-generation tensor cores: C = A B^T, bf16 operands, fp32
 // accumulation in tensor memory, with the decoder-layer epilogues fused:
-//   EPI_QKV    - split into q / k / v, RoPE on q and k at each row's position,
+//   EPI_QKV    - optional bias, split into q / k / v, RoPE on q and k at each row's position,
 //                q to a dense buffer, k / v to (optionally scattered) cache rows;
 //   EPI_RESID  - x += C into the fp32 residual stream (O-proj and down-proj);
 //   EPI_SWIGLU - the B tile holds 128 gate rows and 128 up rows; writes
@@ -58,6 +58,19 @@ KVB_DEV void store16_bf16(uint16_t* dst, const float* v) {
     b.z = pack_bf16(v[12], v[13]); b.w = pack_bf16(v[14], v[15]);
     reinterpret_cast<uint4*>(dst)[0] = a;
     reinterpret_cast<uint4*>(dst)[1] = b;
+}
+
+// x[i] += b[i] for 16 fp32 accumulator words; b is 16-byte aligned
+KVB_DEV void add_bias16(uint32_t* x, const float* b) {
+    const float4* b4 = reinterpret_cast<const float4*>(b);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+        const float4 t = __ldg(b4 + v);
+        x[4 * v] = __float_as_uint(__uint_as_float(x[4 * v]) + t.x);
+        x[4 * v + 1] = __float_as_uint(__uint_as_float(x[4 * v + 1]) + t.y);
+        x[4 * v + 2] = __float_as_uint(__uint_as_float(x[4 * v + 2]) + t.z);
+        x[4 * v + 3] = __float_as_uint(__uint_as_float(x[4 * v + 3]) + t.w);
+    }
 }
 
 template <int EPI, int HD>
@@ -205,6 +218,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                             tmem_ld16(tcol + HD / 2 + c * 16, x2);
                             tmem_ld_wait();
                             if (valid) {
+                                if (p.bias) {
+                                    add_bias16(x1, p.bias + colL + c * 16);
+                                    add_bias16(x2, p.bias + colL + HD / 2 + c * 16);
+                                }
                                 float y1[16], y2[16];
                                 const float4* cp = reinterpret_cast<const float4*>(crow + c * 16);
                                 const float4* sp = reinterpret_cast<const float4*>(srow + c * 16);
@@ -232,6 +249,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                             tmem_ld16(tcol + c * 16, x1);
                             tmem_ld_wait();
                             if (valid) {
+                                if (p.bias) add_bias16(x1, p.bias + colL + c * 16);
                                 float y[16];
 #pragma unroll
                                 for (int i = 0; i < 16; ++i) y[i] = __uint_as_float(x1[i]);

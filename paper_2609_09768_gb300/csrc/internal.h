@@ -50,6 +50,7 @@ struct GemmParams {
     const int32_t* rope_pos;
     const float* cos_t;
     const float* sin_t;
+    const float* bias;            // fp32 bias of the [q | k | v] columns (added before RoPE), or NULL
     // EPI_RESID: x[r][c] += acc
     float* x;
     int64_t ldx;
@@ -116,6 +117,7 @@ enum GemvMode { GEMV_QKV = 0, GEMV_RESID = 1, GEMV_SWIGLU = 2 };
 struct GemvArgs {
     const uint16_t* W;            // [N][K] bf16 (QKV: w_qkv; SwiGLU: gate rows)
     const uint16_t* W2;           // SwiGLU: up rows [N][K]
+    const float* bias;            // QKV: fp32 bias per w_qkv row (added before RoPE), or NULL
     int64_t N;                    // output rows (RESID, SWIGLU)
     int K;
     const uint16_t* a;            // RESID: bf16 input row [K]

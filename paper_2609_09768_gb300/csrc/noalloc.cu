@@ -73,6 +73,7 @@ extern "C" kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, cons
         if (!p || !aligned16(p)) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: NULL or misaligned pointer");
     if (status_out && !aligned16(status_out))
         return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: status_out not 16-byte aligned");
+    if (w->b_qkv && !aligned16(w->b_qkv)) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: b_qkv not 16-byte aligned");
 
     void* scratch = nullptr;
     kvb_status s = scratch_address(&scratch);
@@ -88,6 +89,6 @@ extern "C" kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, cons
     p.M = m; p.N = QD + 2 * KVD; p.K = H; p.epi = EPI_QKV;
     p.col_base = 0; p.q_dim = QD; p.kv_dim = KVD; p.head_dim = D;
     p.q_out = q_out; p.k_out = k_out; p.v_out = v_out; p.kv_dst = kv_dst; p.rope_pos = rope_pos;
-    p.cos_t = rope->cos; p.sin_t = rope->sin; p.status = status_out;
+    p.cos_t = rope->cos; p.sin_t = rope->sin; p.bias = w->b_qkv; p.status = status_out;
     return launch_gemm(p, a, H, w->w_qkv, H, nullptr, st);
 }

@@ -30,18 +30,19 @@ class KvbError(RuntimeError):
 STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "CUDA error", 4: "device wait timed out",
           5: "workspace too small"}
 KVB_OK, KVB_ERR_INVALID_ARG, KVB_ERR_UNSUPPORTED, KVB_ERR_CUDA, KVB_ERR_TIMEOUT, KVB_ERR_WORKSPACE = range(6)
+KVB_ROPE_PLAIN, KVB_ROPE_LLAMA3, KVB_ROPE_YARN = range(3)
 
 
 class Config(C.Structure):
     _fields_ = [("hidden", c_i32), ("n_q_heads", c_i32), ("n_kv_heads", c_i32), ("head_dim", c_i32),
                 ("mlp_dim", c_i32), ("n_layers", c_i32), ("vocab", c_i32), ("rms_eps", c_f32),
-                ("rope_theta", c_f32), ("rope_llama3", c_i32), ("rs_factor", c_f32), ("rs_low", c_f32),
+                ("rope_theta", c_f32), ("rope_scaling", c_i32), ("rs_factor", c_f32), ("rs_low", c_f32),
                 ("rs_high", c_f32), ("rs_orig_ctx", c_i32)]
 
 
 class LayerWeights(C.Structure):
     _fields_ = [("attn_norm", c_vp), ("w_qkv", c_vp), ("w_o", c_vp), ("mlp_norm", c_vp), ("w_gate", c_vp),
-                ("w_up", c_vp), ("w_down", c_vp)]
+                ("w_up", c_vp), ("w_down", c_vp), ("b_qkv", c_vp)]
 
 
 class ModelStruct(C.Structure):
@@ -72,6 +73,7 @@ _SIGS = {
     "kvb_last_error": (C.c_char_p, []),
     "kvb_version": (c_i32, []),
     "kvb_rope_table_fill": (c_i32, [P(Config), c_i64, c_vp, c_vp]),
+    "kvb_attention_scale": (c_i32, [P(Config), P(c_f32)]),
     "kvb_rope_realign": (c_i32, [P(Config), P(RopeTableStruct), c_vp, c_vp, c_i64, c_vp, c_vp, c_i64, c_i32, c_i32,
                                  c_vp, c_i32, c_i64, c_vp]),
     "kvb_hkvd_workspace_size": (c_sz, [c_i64]),
@@ -168,6 +170,13 @@ def rope_table_fill(cfg: Config, max_pos: int) -> Tuple[np.ndarray, np.ndarray]:
     return cos, sin
 
 
+def attention_scale(cfg: Config) -> float:
+    """The q.k factor of every attention kernel (1/sqrt(D), times YaRN's temperature)."""
+    out = c_f32(0.0)
+    _call("kvb_attention_scale", C.byref(cfg), C.byref(out))
+    return out.value
+
+
 class RopeTable:
     """Device cos/sin tables [max_pos][D/2] (fp32) and the struct pointing at them."""
 
@@ -184,7 +193,7 @@ def layer_struct(lw: Dict[str, torch.Tensor]) -> LayerWeights:
     return LayerWeights(_ptr(lw["attn_norm"], torch.float32, "attn_norm"), _ptr(lw["w_qkv"], torch.bfloat16, "w_qkv"),
                         _ptr(lw["w_o"], torch.bfloat16, "w_o"), _ptr(lw["mlp_norm"], torch.float32, "mlp_norm"),
                         _ptr(lw["w_gate"], torch.bfloat16, "w_gate"), _ptr(lw["w_up"], torch.bfloat16, "w_up"),
-                        _ptr(lw["w_down"], torch.bfloat16, "w_down"))
+                        _ptr(lw["w_down"], torch.bfloat16, "w_down"), _ptr(lw.get("b_qkv"), torch.float32, "b_qkv"))
 
 
 class Model:

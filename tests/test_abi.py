@@ -45,12 +45,41 @@ def test_status_strings_and_version(kvb):
 
 
 def test_rope_table_matches_oracle(kvb):
-    for shape in (synth.TINY, synth.LLAMA8B):
+    for shape in (synth.TINY, synth.LLAMA8B, synth.YARN_GQA7_TINY, synth.YARN_GQA7):
         cfg = kvb.config(shape)
         cos, sin = kvb.rope_table_fill(cfg, 130000)
         pos = np.array([0, 1, 2, 511, 8191, 8192, 65537, 124031, 129999])
         c, s = llama.rope_cos_sin(Shape.of(shape), pos)
         assert np.max(np.abs(cos[pos] - c)) < 1e-6 and np.max(np.abs(sin[pos] - s)) < 1e-6
+
+
+def test_attention_scale_matches_oracle(kvb):
+    """1/sqrt(D), times YaRN's (0.1 ln s + 1)^2 for the YaRN shapes."""
+    for shape in (synth.TINY, synth.LLAMA8B, synth.YARN_GQA7_TINY, synth.YARN_GQA7):
+        got = kvb.attention_scale(kvb.config(shape))
+        assert abs(got - llama.logit_scale(Shape.of(shape))) <= 1e-7 * got
+    assert kvb.attention_scale(kvb.config(synth.YARN_GQA7)) > 1.0 / np.sqrt(128) * 1.2
+
+
+def test_config_validation_of_rope_scaling_and_groups(kvb):
+    L = kvb.lib()
+    n = C.c_size_t(0)
+    cfg = kvb.config(synth.YARN_GQA7)           # seven q heads per kv head: accepted
+    assert L.kvb_workspace_size(C.byref(cfg), 100, C.byref(n)) == kvb.KVB_OK
+    assert L.kvb_decode_workspace_size(C.byref(cfg), 100, C.byref(n)) == kvb.KVB_OK
+    bad = kvb.config(synth.YARN_GQA7)
+    bad.rope_scaling = 3
+    assert L.kvb_workspace_size(C.byref(bad), 100, C.byref(n)) == kvb.KVB_ERR_INVALID_ARG
+    bad = kvb.config(synth.YARN_GQA7)
+    bad.rs_factor = 0.5                         # YaRN extends the context: s >= 1
+    assert L.kvb_workspace_size(C.byref(bad), 100, C.byref(n)) == kvb.KVB_ERR_INVALID_ARG
+    bad = kvb.config(synth.YARN_GQA7)
+    bad.rs_high = bad.rs_low
+    assert L.kvb_workspace_size(C.byref(bad), 100, C.byref(n)) == kvb.KVB_ERR_INVALID_ARG
+    three = kvb.config(synth.LLAMA8B)           # 3 q heads per kv head: prefill yes, decode not built
+    three.n_q_heads, three.n_kv_heads = 24, 8
+    assert L.kvb_workspace_size(C.byref(three), 100, C.byref(n)) == kvb.KVB_OK
+    assert L.kvb_decode_workspace_size(C.byref(three), 100, C.byref(n)) == kvb.KVB_ERR_UNSUPPORTED
 
 
 def test_workspace_size_grows_with_rows(kvb):

@@ -34,6 +34,8 @@ def dev(t):
     (L8B, 3000, [0, 1, 255, 256, 257, 2999]),      # split edges, a single key, the last row
     (TINY, 600, [0, 300, 599]),
     (L8B, 124160, [124031]),                        # the headline length (124,032 rows)
+    (synth.YARN_GQA7, 3000, [0, 1, 1023, 1024, 2999]),   # 7 q heads per kv head, YaRN temperature
+    (synth.YARN_GQA7_TINY, 600, [0, 300, 599]),
 ])
 def test_decode_attention_matches_oracle(kvb, shape, n_rows, positions):
     cfg = kvb.config(shape)
@@ -129,7 +131,7 @@ class DecodeCase:
 _CASES = {}
 
 
-@pytest.fixture(scope="module", params=["tiny", "l8b_1layer"])
+@pytest.fixture(scope="module", params=["tiny", "l8b_1layer", "yarn_tiny", "yarn_2l"])
 def case(request, kvb):
     if request.param not in _CASES:
         _CASES[request.param] = DecodeCase(kvb, synth.WORKLOADS[request.param])

@@ -13,6 +13,8 @@ pytestmark = pytest.mark.gpu
 
 TINY = synth.TINY
 L8B = synth.LLAMA8B.with_layers(2)
+YT = synth.YARN_GQA7_TINY            # YaRN, 7 q heads per kv head, q/k/v bias
+Y2 = synth.YARN_GQA7
 
 
 @pytest.fixture(scope="module")
@@ -99,7 +101,7 @@ def test_hkvd_exact_ties_take_lowest_index(kvb):
 # ------------------------------------------------------------------------------------------ QKV GEMM
 
 @pytest.mark.parametrize("shape,m,n_src", [(TINY, 108, 544), (L8B, 640, 3904), (L8B, 1, 7), (TINY, 129, 300),
-                                           (L8B, 300, 300)])
+                                           (L8B, 300, 300), (YT, 108, 544), (Y2, 640, 3904), (Y2, 1, 7)])
 def test_gather_rmsnorm_qkv_matches_oracle(kvb, shape, m, n_src):
     cfg = kvb.config(shape)
     lw = synth.make_layer_weights(shape, 1, seed=5)
@@ -150,7 +152,8 @@ def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
     return out.cpu(), ref.reshape(m, -1), float(np.sqrt(np.mean(np64(v) ** 2)))
 
 
-@pytest.mark.parametrize("shape,n_kv", [(TINY, 544), (L8B, 3904), (TINY, 1), (L8B, 130), (L8B, 129)])
+@pytest.mark.parametrize("shape,n_kv", [(TINY, 544), (L8B, 3904), (TINY, 1), (L8B, 130), (L8B, 129), (YT, 544),
+                                        (Y2, 3904), (Y2, 19), (YT, 1)])
 def test_attention_dense_causal(kvb, shape, n_kv):
     out, ref, vs = _attn_case(kvb, shape, n_kv, list(range(n_kv)))
     e = assert_close_rel(out, ref, "dense causal attention", scale=vs)
@@ -158,7 +161,7 @@ def test_attention_dense_causal(kvb, shape, n_kv):
 
 
 @pytest.mark.parametrize("shape,n_kv,m", [(TINY, 544, 108), (L8B, 3904, 640), (L8B, 3904, 33), (L8B, 5000, 1),
-                                          (TINY, 200, 3)])
+                                          (TINY, 200, 3), (Y2, 3904, 640), (YT, 544, 37)])
 def test_attention_sparse_rows(kvb, shape, n_kv, m):
     g = np.random.default_rng(m)
     rows = np.sort(g.choice(n_kv, size=m, replace=False))
@@ -169,7 +172,8 @@ def test_attention_sparse_rows(kvb, shape, n_kv, m):
 
 
 @pytest.mark.parametrize("shape,starts", [(TINY, [0, 128, 256, 384, 512]), (L8B, [0, 480, 960, 1440]),
-                                          (TINY, [0, 5, 140, 141, 300])])
+                                          (TINY, [0, 5, 140, 141, 300]), (Y2, [0, 480, 960, 1440]),
+                                          (YT, [0, 5, 140, 141, 300])])
 def test_attention_block_diagonal(kvb, shape, starts):
     n = starts[-1]
     lo = np.concatenate([[starts[c]] * (starts[c + 1] - starts[c]) for c in range(len(starts) - 1)])
@@ -180,7 +184,7 @@ def test_attention_block_diagonal(kvb, shape, starts):
 
 # ------------------------------------------------------------------------------------------ MLP half
 
-@pytest.mark.parametrize("shape,m", [(TINY, 108), (L8B, 640), (L8B, 1), (TINY, 300)])
+@pytest.mark.parametrize("shape,m", [(TINY, 108), (L8B, 640), (L8B, 1), (TINY, 300), (Y2, 640), (YT, 108)])
 def test_mlp_rows_matches_oracle(kvb, shape, m):
     cfg = kvb.config(shape)
     lw = synth.make_layer_weights(shape, 0, seed=9)

@@ -1,6 +1,7 @@
 """End-to-end parity of the whole path through the C ABI against the float64 oracle:
 per-chunk caches, the dense prefill (the r = 1 comparator) and the selective
-prefill, on the tiny model and the Llama-3.1-8B-shaped 2-layer model."""
+prefill, on the tiny model, the Llama-3.1-8B-shaped 2-layer model and two YaRN models
+with seven q heads per kv head and a q/k/v bias."""
 import numpy as np
 import pytest
 import torch
@@ -103,7 +104,7 @@ class Case:
 _CASES = {}
 
 
-@pytest.fixture(scope="module", params=["tiny", "l8b_1layer", "tiny_sep", "l8b_1layer_sep"])
+@pytest.fixture(scope="module", params=["tiny", "l8b_1layer", "tiny_sep", "l8b_1layer_sep", "yarn_tiny", "yarn_2l"])
 def case(request, kvb):
     if request.param not in _CASES:
         _CASES[request.param] = Case(kvb, synth.WORKLOADS[request.param])

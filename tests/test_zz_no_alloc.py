@@ -48,7 +48,8 @@ def _run_pair(kvb, shape, m, n_src, seed):
     return outs
 
 
-@pytest.mark.parametrize("shape,m,n_src", [(synth.LLAMA8B.with_layers(2), 1024, 3904), (synth.TINY, 300, 544)])
+@pytest.mark.parametrize("shape,m,n_src", [(synth.LLAMA8B.with_layers(2), 1024, 3904), (synth.TINY, 300, 544),
+                                           (synth.YARN_GQA7, 700, 3904)])
 def test_noalloc_matches_workspace_entry_point_on_two_calls(kvb, shape, m, n_src):
     for seed, mm in ((21, m), (22, m // 3 + 1)):       # two calls in a row, the second smaller
         (q, kc, vc), (q2, kc2, vc2) = _run_pair(kvb, shape, mm, n_src, seed)
