@@ -37,7 +37,7 @@ METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % 
 # size (18,713 rows over a 124,032-row cache), from the ncu capture summarised in
 # profiles/attn_kernel_sparse_m18713_nkv124032.md; valid only for the kernel sources it
 # was taken on (sha1 prefixes of attn.cu and common.cuh), otherwise reported as null.
-ATTN_TRAFFIC = {"bytes": 8.171074e9 + 0.141687e9, "sha1": {"attn.cu": "53c3e0fbf4ab", "common.cuh": "1bea4aeef0d1"}}
+ATTN_TRAFFIC = {"bytes": 8.170141e9 + 0.141452e9, "sha1": {"attn.cu": "4d66f8ec5f4a", "common.cuh": "1bea4aeef0d1"}}
 
 
 def attn_traffic():
@@ -57,6 +57,9 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="l8b_124k")
+    ap.add_argument("--model-config", default=None,
+                    help="JSON model configuration (published-checkpoint layout) whose shape replaces the "
+                         "workload's model; chunk layout, query and r stay the workload's")
     ap.add_argument("--r", type=float, default=None)
     ap.add_argument("--r1-steps", type=int, default=1, help="timed steps of the r = 1.0 comparator (0: skip)")
     ap.add_argument("--e2e-steps", type=int, default=2, help="timed end-to-end steps (0: skip)")
@@ -603,6 +606,12 @@ def main():
     args = parse()
     from paper_2609_09768_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
+    if args.model_config:
+        import dataclasses
+        with open(args.model_config) as fh:
+            shape = synth.shape_from_config(json.load(fh))
+        name = os.path.splitext(os.path.basename(args.model_config))[0]
+        wl = dataclasses.replace(wl, shape=shape, name=f"{name}-{shape.n_layers}L-{wl.n_chunks}x{wl.chunk_len}+{wl.n_query}")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":

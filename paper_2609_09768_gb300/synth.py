@@ -29,7 +29,7 @@ from typing import Dict, List, Optional, Sequence
 import torch
 
 __all__ = [
-    "ModelShape", "Workload", "SHAPES", "WORKLOADS", "tensor_seed",
+    "ModelShape", "Workload", "SHAPES", "WORKLOADS", "tensor_seed", "shape_from_config",
     "make_layer_weights", "make_embed", "make_lm_head", "make_model", "make_tokens",
     "chunk_starts_equal", "separator_layout", "separator_ids", "randn_bf16",
 ]
@@ -153,7 +153,37 @@ WORKLOADS: Dict[str, Workload] = {
     # YaRN RoPE, seven q heads per kv head, q/k/v bias
     "yarn_tiny": Workload("yarn-gqa7-tiny-2L-4x128+32", YARN_GQA7_TINY, 4, 128, 32),
     "yarn_2l": Workload("yarn-gqa7-2L-8x480+64", YARN_GQA7, 8, 480, 64),
+    "yarn_124k": Workload("yarn-gqa7-32L-242x512+128", YARN_GQA7.with_layers(32), 242, 512, 128),
 }
+
+
+def shape_from_config(cfg: dict) -> ModelShape:
+    """A ModelShape from a model configuration in the common JSON layout of published
+    decoder checkpoints (hidden_size, num_attention_heads, num_key_value_heads,
+    intermediate_size, num_hidden_layers, vocab_size, rms_norm_eps, rope_theta and an
+    optional rope_scaling block of type "llama3" or "yarn").  The q/k/v bias is taken from
+    "attention_bias" when present, else from a "qkv_bias" key (False if neither).  YaRN's
+    ramp bounds default to alpha = 1, beta = 32 when the block does not give them."""
+    H = int(cfg["hidden_size"])
+    Hq = int(cfg["num_attention_heads"])
+    Hkv = int(cfg.get("num_key_value_heads", Hq))
+    D = int(cfg.get("head_dim") or H // Hq)
+    kw = {}
+    rs = cfg.get("rope_scaling") or {}
+    kind = (rs.get("rope_type") or rs.get("type") or "default").lower()
+    if kind == "llama3":
+        kw = dict(rope_scaling=1, rs_factor=float(rs["factor"]), rs_low=float(rs["low_freq_factor"]),
+                  rs_high=float(rs["high_freq_factor"]), rs_orig_ctx=int(rs["original_max_position_embeddings"]))
+    elif kind == "yarn":
+        kw = dict(rope_scaling=2, rs_factor=float(rs["factor"]), rs_low=float(rs.get("beta_slow", 1.0)),
+                  rs_high=float(rs.get("beta_fast", 32.0)), rs_orig_ctx=int(rs["original_max_position_embeddings"]))
+    elif kind not in ("default", "none"):
+        raise ValueError(f"rope_scaling type {kind!r} is not supported")
+    bias = bool(cfg.get("attention_bias", cfg.get("qkv_bias", False)))
+    return ModelShape(hidden=H, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=D, mlp_dim=int(cfg["intermediate_size"]),
+                      n_layers=int(cfg["num_hidden_layers"]), vocab=int(cfg["vocab_size"]),
+                      rms_eps=float(cfg.get("rms_norm_eps", 1e-5)), rope_theta=float(cfg.get("rope_theta", 10000.0)),
+                      qkv_bias=bias, **kw)
 
 
 def tensor_seed(seed: int, layer: int, name: str) -> int:

@@ -127,3 +127,25 @@ def test_binding_fails_loudly_without_library(monkeypatch):
     monkeypatch.setattr(kvblend, "LIB", "/nonexistent/libkvblend.so")
     with pytest.raises(RuntimeError, match="not built"):
         kvblend.lib()
+
+
+def test_shape_from_published_config_layout():
+    """The config reader maps the common checkpoint JSON layout onto ModelShape (values here
+    are made up for the test)."""
+    base = {"hidden_size": 1792, "num_attention_heads": 14, "num_key_value_heads": 2, "intermediate_size": 4864,
+            "num_hidden_layers": 3, "vocab_size": 5000, "rms_norm_eps": 1e-6, "rope_theta": 1e6}
+    s = synth.shape_from_config(dict(base, rope_scaling={"type": "yarn", "factor": 4.0,
+                                                         "original_max_position_embeddings": 2048}, qkv_bias=True))
+    assert (s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.mlp_dim, s.n_layers, s.vocab) == \
+        (1792, 14, 2, 128, 4864, 3, 5000)
+    assert (s.rope_scaling, s.rs_factor, s.rs_low, s.rs_high, s.rs_orig_ctx, s.qkv_bias) == (2, 4.0, 1.0, 32.0, 2048, True)
+    assert s == synth.YARN_GQA7.with_layers(3).__class__(**{**synth.YARN_GQA7.__dict__, "n_layers": 3, "vocab": 5000})
+    l3 = synth.shape_from_config(dict(base, rope_scaling={"rope_type": "llama3", "factor": 8.0, "low_freq_factor": 1.0,
+                                                          "high_freq_factor": 4.0,
+                                                          "original_max_position_embeddings": 8192},
+                                      attention_bias=False))
+    assert (l3.rope_scaling, l3.rs_factor, l3.rs_low, l3.rs_high, l3.rs_orig_ctx, l3.qkv_bias) == (1, 8.0, 1.0, 4.0, 8192, False)
+    plain = synth.shape_from_config(dict(base, head_dim=64))
+    assert plain.rope_scaling == 0 and plain.head_dim == 64
+    with pytest.raises(ValueError):
+        synth.shape_from_config(dict(base, rope_scaling={"type": "dynamic", "factor": 2.0}))
