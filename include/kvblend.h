@@ -73,8 +73,7 @@ enum {
 };
 
 /* Model shape and RoPE settings.  Hq must be a multiple of Hkv; any group size
- * Hq/Hkv <= 128 runs in the prefill, the decode attention is built for group sizes
- * 1, 2, 4, 7 and 8. */
+ * Hq/Hkv <= 128 runs in the prefill, group sizes up to 8 in the decode. */
 typedef struct kvb_config {
     int32_t hidden, n_q_heads, n_kv_heads, head_dim, mlp_dim, n_layers, vocab;
     float rms_eps;

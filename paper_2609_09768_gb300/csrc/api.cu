@@ -961,9 +961,8 @@ static kvb_status check_decode(const kvb_config* cfg, int64_t max_pos) {
     const int64_t qd = (int64_t)cfg->n_q_heads * cfg->head_dim;
     if (cfg->hidden > KVB_DECODE_MAX_K || cfg->mlp_dim > KVB_DECODE_MAX_K || qd > KVB_DECODE_MAX_K)
         return fail(KVB_ERR_UNSUPPORTED, "decode: hidden, mlp_dim and Hq*D must be at most %d", KVB_DECODE_MAX_K);
-    const int G = cfg->n_q_heads / cfg->n_kv_heads;
-    if (G != 1 && G != 2 && G != 4 && G != 7 && G != 8)
-        return fail(KVB_ERR_UNSUPPORTED, "decode: %d q heads per kv head not built (1, 2, 4, 7, 8)", G);
+    if (cfg->n_q_heads / cfg->n_kv_heads > 8)
+        return fail(KVB_ERR_UNSUPPORTED, "decode: at most 8 q heads per kv head (%d)", cfg->n_q_heads / cfg->n_kv_heads);
     return KVB_OK;
 }
 

@@ -12,13 +12,12 @@
 //                       q and the cache's K/V row `pos` (V as bf16-rounded fp16, like the
 //                       prefill); the residual mode adds into x; SwiGLU computes gate and
 //                       up rows in one warp
-//   decode_attn       - split-KV attention of the new row over cache rows [0, pos]:
-//                       one warp per split of 128 keys and kv head, lanes over head
-//                       dims; the G q heads sharing the kv head (padded to a power of
-//                       two GP) and 32/GP keys give 32 partial dot products per step, summed with one 31-shuffle
-//                       reduce-scatter; online softmax per head in fp32; the next
-//                       step's K/V loads are issued before this step's arithmetic; the 8
-//                       warps of a CTA merge their (max, sum, O) in shared memory
+//   decode_attn       - split-KV attention of the new row over cache rows [0, pos]: one
+//                       warp per split of 128 rows of one kv head, K/V tiles of 16 rows
+//                       streamed by TMA into a per-warp ring, S^T = K Q^T and O^T += V^T P^T
+//                       on mma.sync tiles with the group's q heads as the 8 columns, online
+//                       softmax per head in fp32; the 4 warps of a CTA merge their
+//                       (max, sum, O) in shared memory
 //   decode_combine    - log-sum-exp merge of the CTA partials -> bf16 attention output
 //   decode_finish     - tokens[pos + 1] = argmax, pos += 1
 // The position and the token live in device memory, so a step needs no host value that
@@ -31,8 +30,6 @@ namespace kvb {
 namespace {
 
 constexpr int GEMV_THREADS = 256;
-constexpr int GEMV_BATCH = 8;
-constexpr int ATT_THREADS = 256;             // 8 warps = 8 splits of one kv head
 
 KVB_DEV bool pos_ok(const int32_t* pos_ptr, int64_t max_pos, int* status, int& pos) {
     pos = *pos_ptr;
@@ -200,200 +197,291 @@ gemv_kernel(const GemvArgs p) {
     }
 }
 
-// Unpack one lane's DPL head dims of a key (bf16) or value (fp16) row from raw words.
-template <int DPL>
-struct RowBits {
-    uint32_t w[DPL / 2];
+// ---------------------------------------------------------------- decode attention
+//
+// One CTA = DA_WARPS warps of one kv head; warp w takes the split of
+// KVB_DECODE_KEYS_PER_SPLIT cache rows starting at (blockIdx.x * DA_WARPS + w) * split and
+// streams it through its own ring of DA_STAGES stages of 16 rows (K and V tiles loaded by
+// TMA, 128-byte swizzle).  Per stage, with the G <= 8 q heads of the group as the 8
+// columns of mma.sync m16n8k16 tiles (columns G..7 are zero q heads, never written out):
+//   S^T [16 keys x 8 heads] = K [16 x D] . Q^T            (bf16, fp32 accumulate)
+//   online softmax per head (column) in the log2 domain;
+//   P^T as the B operand: fp16 pairs of the accumulator rows transposed by movmatrix,
+//       as an fp16 head plus an fp16 remainder (~22-bit weights);
+//   O^T [D x 8 heads] += V^T [D x 16 keys] . P^T          (fp16, V^T via ldmatrix.trans)
+// so a stage costs about 60 warp instructions for 8 KB of K/V (D = 128), and the kernel is
+// bound by the TMA stream.  The warps' (max, sum, O) are merged in shared memory and the
+// CTA writes one partial per q head for decode_combine_kernel.
+
+constexpr int DA_WARPS = 4;
+constexpr int DA_THREADS = 32 * DA_WARPS;
+constexpr int DA_STAGE_KEYS = 16;
+constexpr int DA_STAGES = 3;
+constexpr int DA_KEYS_PER_CTA = KVB_DECODE_KEYS_PER_SPLIT * DA_WARPS;
+constexpr float DA_P_SHIFT = 15.f;           // softmax weights carried as p * 2^15
+
+template <int D>
+struct DaSmem {
+    static constexpr int NB = D / 64;                    // 64-column (128-byte) boxes per row
+    static constexpr int BOX = DA_STAGE_KEYS * 128;      // one box: 16 rows x 128 bytes
+    static constexpr int STAGE = 2 * NB * BOX;           // K boxes, then V boxes
+    static constexpr int RING = DA_WARPS * DA_STAGES * STAGE;
+    static constexpr int OFF_BAR = RING;
+    static constexpr int TOTAL = RING + 256 + 1024;      // barriers + flag, 1024-byte alignment slack
+    // merge buffers (o [W][8][D], m and l [W][8], fp32) reuse the ring after the loop
+    static_assert(DA_WARPS * 8 * D * 4 + 2 * DA_WARPS * 8 * 4 <= RING, "merge buffers");
 };
-template <int DPL>
-KVB_DEV RowBits<DPL> load_row(const uint16_t* p) {
-    RowBits<DPL> r;
-    if constexpr (DPL == 4) {
-        const uint2 u = __ldcs(reinterpret_cast<const uint2*>(p));
-        r.w[0] = u.x; r.w[1] = u.y;
-    } else {
-        r.w[0] = __ldcs(reinterpret_cast<const unsigned int*>(p));
-    }
-    return r;
+
+// byte offset of the 16-byte unit `unit` (dims [8 unit, 8 unit + 8)) of row r in a set of
+// 128-byte-swizzled boxes
+template <int D>
+KVB_DEV uint32_t da_off(int r, int unit) {
+    return (uint32_t)((unit >> 3) * DaSmem<D>::BOX + r * 128 + (((unit & 7) ^ (r & 7)) << 4));
 }
 
-// Head slots per kv head: the lane layout pads a group of G q heads to GP slots, a power
-// of two and at least 4 (so that a step covers at most 8 keys and the K/V prefetch fits in
-// registers); the padding heads have q = 0 and are never written out.
-__host__ __device__ constexpr int pad_pow2(int g) { return g <= 4 ? 4 : 8; }
+KVB_DEV void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr)
+                 : "memory");
+}
+KVB_DEV void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr)
+                 : "memory");
+}
+KVB_DEV void mma16816_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                           uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+KVB_DEV void mma16816_f16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                          uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+KVB_DEV uint32_t movmatrix_trans(uint32_t a) {
+    uint32_t d;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+    return d;
+}
 
-// One CTA = eight consecutive splits of KVB_DECODE_KEYS_PER_SPLIT cache rows for kv head
-// blockIdx.y, one warp per split; the warps' partial results are merged in shared memory
-// and the CTA writes one partial (max, sum, O) per q head.
-template <int D, int G>
-__global__ void __launch_bounds__(ATT_THREADS, 2)
-decode_attn_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ kc, const uint16_t* __restrict__ vc,
-                   int Hkv, const int32_t* __restrict__ pos_ptr, int64_t max_pos, int n_blocks, float scale_log2,
-                   float* __restrict__ pm, float* __restrict__ pl, float* __restrict__ po, int* status) {
-    constexpr int DPL = D / 32;      // head dims per lane
-    constexpr int GP = pad_pow2(G);  // head slots
-    static_assert(G >= 1 && G <= 8, "group size");
-    constexpr int KS = 32 / GP;      // keys per step: KS * GP = 32 partial dot products
-    constexpr int WARPS = ATT_THREADS / 32;
-    __shared__ float sm_m[WARPS][GP], sm_l[WARPS][GP];
-    __shared__ float sm_o[WARPS][GP][D];
+template <int D>
+__global__ void __launch_bounds__(DA_THREADS, 2)
+decode_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                   const uint16_t* __restrict__ q, int G, int Hkv, const int32_t* __restrict__ pos_ptr,
+                   int64_t max_pos, int n_blocks, float sl2, float* __restrict__ pm, float* __restrict__ pl,
+                   float* __restrict__ po, int* status) {
+    using S = DaSmem<D>;
+    constexpr int NB = S::NB;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);          // [DA_WARPS][DA_STAGES]
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + DA_WARPS * DA_STAGES);
     int pos;
     if (!pos_ok(pos_ptr, max_pos, status, pos)) return;
     if ((int)blockIdx.x >= n_blocks) return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int g = blockIdx.y;
-    const int Hq = Hkv * G;
-    const int64_t start = ((int64_t)blockIdx.x * WARPS + warp) * KVB_DECODE_KEYS_PER_SPLIT;
+    const int kvh = blockIdx.y;
+    const int g8 = lane >> 2, t4 = lane & 3;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < DA_WARPS * DA_STAGES; ++i) mbar_init(&bars[i], 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (threadIdx.x == 32) { prefetch_tmap(&tmK); prefetch_tmap(&tmV); }
+    __syncthreads();
+
+    const int64_t start = ((int64_t)blockIdx.x * DA_WARPS + warp) * KVB_DECODE_KEYS_PER_SPLIT;
     int64_t end = start + KVB_DECODE_KEYS_PER_SPLIT;
     if (end > (int64_t)pos + 1) end = (int64_t)pos + 1;
-
-    // q of the G heads (zero for the padding slots) in shared memory (registers go to the
-    // K/V prefetch)
-    __shared__ __align__(16) float qs[GP][D];
-    __shared__ __align__(16) float sp[ATT_THREADS / 32][32];   // per warp: this step's weights
-    __shared__ float sa[ATT_THREADS / 32][GP];                  // per warp: rescale factor per head
-    for (int i = threadIdx.x; i < GP * D; i += ATT_THREADS)
-        qs[i / D][i % D] = i < G * D ? bf16_to_f(q[(g * G) * D + i]) : 0.f;
-    __syncthreads();
-    float o[GP][DPL];
+    const int n_st = start < end ? (int)((end - start + DA_STAGE_KEYS - 1) / DA_STAGE_KEYS) : 0;
+    uint8_t* ring = smem + warp * DA_STAGES * S::STAGE;
+    uint64_t* wbar = bars + warp * DA_STAGES;
+    auto issue = [&](int st) {            // lane 0: K and V rows of stage st into its slot
+        uint8_t* dst = ring + (st % DA_STAGES) * S::STAGE;
+        uint64_t* b = wbar + st % DA_STAGES;
+        const int y = (int)(start + (int64_t)st * DA_STAGE_KEYS);
+        mbar_expect_tx(b, S::STAGE);
 #pragma unroll
-    for (int h = 0; h < GP; ++h)
+        for (int c = 0; c < NB; ++c) tma_load_2d(dst + c * S::BOX, &tmK, b, kvh * D + c * 64, y);
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) o[h][e] = 0.f;
-    float m_run = -INFINITY, l_run = 0.f;    // of head slot lane % GP
-
-    const int64_t row_stride = (int64_t)Hkv * D;
-    const uint16_t* kbase = kc + (int64_t)g * D + lane * DPL;
-    const uint16_t* vbase = vc + (int64_t)g * D + lane * DPL;
-    RowBits<DPL> ck[KS], cv[KS], nk[KS], nv[KS];
-    auto fetch = [&](int64_t k0, RowBits<DPL>* kr, RowBits<DPL>* vr) {
-#pragma unroll
-        for (int k = 0; k < KS; ++k) {
-            if (k0 + k < end) {
-                kr[k] = load_row<DPL>(kbase + (k0 + k) * row_stride);
-                vr[k] = load_row<DPL>(vbase + (k0 + k) * row_stride);
-            } else {
-#pragma unroll
-                for (int i = 0; i < DPL / 2; ++i) { kr[k].w[i] = 0u; vr[k].w[i] = 0u; }
-            }
-        }
+        for (int c = 0; c < NB; ++c) tma_load_2d(dst + (NB + c) * S::BOX, &tmV, b, kvh * D + c * 64, y);
     };
-    if (start < end) fetch(start, ck, cv);
-    for (int64_t k0 = start; k0 < end; k0 += KS) {
-        // loads of the next step go out before this step's arithmetic
-        if (k0 + KS < end) fetch(k0 + KS, nk, nv);
-        float sc[32];
-        {
-            float qv[GP][DPL];   // this lane's head dims of q, once per step
+    int issued = n_st < DA_STAGES ? n_st : DA_STAGES;
+    if (lane == 0)
+        for (int st = 0; st < issued; ++st) issue(st);
+
+    // B operand of S^T = K Q^T: q head g8 of the group (zero columns for g8 >= G), dims
+    // 16 ks + 2 t4 (+1) and 16 ks + 8 + 2 t4 (+1)
+    uint32_t qb[D / 16][2];
+    {
+        const uint32_t* qrow = reinterpret_cast<const uint32_t*>(q + ((int64_t)kvh * G + g8) * D);
 #pragma unroll
-            for (int h = 0; h < GP; ++h) {
-                if constexpr (DPL == 4) {
-                    const float4 t4 = *reinterpret_cast<const float4*>(&qs[h][lane * 4]);
-                    qv[h][0] = t4.x; qv[h][1] = t4.y; qv[h][2] = t4.z; qv[h][3] = t4.w;
-                } else {
-                    const float2 t2 = *reinterpret_cast<const float2*>(&qs[h][lane * 2]);
-                    qv[h][0] = t2.x; qv[h][1] = t2.y;
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < KS; ++k) {
-                float kf[DPL];
-#pragma unroll
-                for (int i = 0; i < DPL / 2; ++i) { kf[2 * i] = bf16_lo(ck[k].w[i]); kf[2 * i + 1] = bf16_hi(ck[k].w[i]); }
-#pragma unroll
-                for (int h = 0; h < GP; ++h) {
-                    float acc = 0.f;
-#pragma unroll
-                    for (int e = 0; e < DPL; ++e) acc = fmaf(qv[h][e], kf[e], acc);
-                    sc[k * GP + h] = acc;
-                }
-            }
+        for (int ks = 0; ks < D / 16; ++ks) {
+            qb[ks][0] = g8 < G ? __ldg(qrow + 8 * ks + t4) : 0u;
+            qb[ks][1] = g8 < G ? __ldg(qrow + 8 * ks + 4 + t4) : 0u;
         }
-        // reduce-scatter: afterwards lane L holds the full dot product of index L
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) {
-#pragma unroll
-            for (int i = 0; i < off; ++i) {
-                const bool upper = (lane & off) != 0;
-                const float send = upper ? sc[i] : sc[i + off];
-                const float keep = upper ? sc[i + off] : sc[i];
-                sc[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
-            }
-        }
-        float t = sc[0] * scale_log2;
-        if (k0 + lane / GP >= end) t = -INFINITY;
-        // online softmax of head slot lane % GP over this step's keys
-        float mx = t;
-#pragma unroll
-        for (int off = GP; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-        const float m_new = fmaxf(m_run, mx);
-        const float alpha = (m_new == -INFINITY) ? 1.f : fast_exp2(m_run - m_new);
-        const float pv = (t == -INFINITY) ? 0.f : fast_exp2(t - m_new);
-        float ps = pv;
-#pragma unroll
-        for (int off = GP; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
-        l_run = l_run * alpha + ps;
-        m_run = m_new;
-        // this step's weights (index key * GP + head) and the heads' rescale factors to every lane
-        __syncwarp();
-        sp[warp][lane] = pv;
-        if (lane < GP) sa[warp][lane] = alpha;
-        __syncwarp();
-#pragma unroll
-        for (int h = 0; h < GP; ++h) {
-            const float ah = sa[warp][h];
-#pragma unroll
-            for (int e = 0; e < DPL; ++e) o[h][e] *= ah;
-        }
-#pragma unroll
-        for (int k = 0; k < KS; ++k) {
-            float vf[DPL];
-#pragma unroll
-            for (int i = 0; i < DPL / 2; ++i) {
-                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&cv[k].w[i]));
-                vf[2 * i] = f.x; vf[2 * i + 1] = f.y;
-            }
-            float pk[GP];   // weights of key k for the GP head slots, vector loads (broadcast)
-            if constexpr (GP % 4 == 0) {
-#pragma unroll
-                for (int h4 = 0; h4 < GP; h4 += 4) {
-                    const float4 t = *reinterpret_cast<const float4*>(&sp[warp][k * GP + h4]);
-                    pk[h4] = t.x; pk[h4 + 1] = t.y; pk[h4 + 2] = t.z; pk[h4 + 3] = t.w;
-                }
-            } else if constexpr (GP == 2) {
-                const float2 t = *reinterpret_cast<const float2*>(&sp[warp][k * GP]);
-                pk[0] = t.x; pk[1] = t.y;
-            } else {
-                pk[0] = sp[warp][k];
-            }
-#pragma unroll
-            for (int h = 0; h < GP; ++h) {
-#pragma unroll
-                for (int e = 0; e < DPL; ++e) o[h][e] = fmaf(pk[h], vf[e], o[h][e]);
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < KS; ++k) { ck[k] = nk[k]; cv[k] = nv[k]; }
     }
-    // merge the warps of this CTA (the G real heads)
+    float o[D / 16][4];
 #pragma unroll
-    for (int h = 0; h < G; ++h)
+    for (int m = 0; m < D / 16; ++m) o[m][0] = o[m][1] = o[m][2] = o[m][3] = 0.f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;     // heads 2 t4 and 2 t4 + 1
+    // this lane's ldmatrix rows: K (A of S^T) and V (A of O^T, transposed)
+    const int mm = lane >> 3;
+    const int rk = ((mm & 1) << 3) | (lane & 7), uk = mm >> 1;
+    const int rv = ((mm >> 1) << 3) | (lane & 7), uv = mm & 1;
+
+    int st = 0;
+    bool ok = true;
+    for (; st < n_st; ++st) {
+        const int slot = st % DA_STAGES;
+        if (!mbar_wait_warp(wbar + slot, (uint32_t)(st / DA_STAGES) & 1, abort_flag, status)) {
+            ok = false;
+            break;
+        }
+        uint8_t* sp = ring + slot * S::STAGE;
+        const uint32_t kb = smem_u32(sp), vb = kb + NB * S::BOX;
+        const int64_t key0 = start + (int64_t)st * DA_STAGE_KEYS;
+        const int nvalid = (int)((end - key0) < DA_STAGE_KEYS ? (end - key0) : DA_STAGE_KEYS);
+        if (nvalid < DA_STAGE_KEYS) {
+            // rows past the current position: zero their V (the cache may hold anything there)
+            uint4* vz = reinterpret_cast<uint4*>(sp + NB * S::BOX);
+            for (int i = lane; i < NB * DA_STAGE_KEYS * 8; i += 32)
+                if (((i >> 3) & (DA_STAGE_KEYS - 1)) >= nvalid) vz[i] = make_uint4(0u, 0u, 0u, 0u);
+            __syncwarp();
+        }
+        // S^T: rows = keys g8 and g8 + 8, columns = heads 2 t4 and 2 t4 + 1.  Every 16-dim
+        // slice gets its own accumulator (one MMA from zero: the tensor core's sum of 16 exact
+        // bf16 products) and the slices are added in fp32 afterwards, instead of chaining the
+        // MMAs through one accumulator whose running sum the tensor core rounds at every step.
+        float sk[D / 16][4];
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) sm_o[warp][h][lane * DPL + e] = o[h][e];
-    if (lane < G) { sm_m[warp][lane] = m_run; sm_l[warp][lane] = l_run; }
+        for (int ks = 0; ks < D / 16; ++ks) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(kb + da_off<D>(rk, 2 * ks + uk), a0, a1, a2, a3);
+            sk[ks][0] = sk[ks][1] = sk[ks][2] = sk[ks][3] = 0.f;
+            mma16816_bf16(sk[ks], a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+        }
+        float sacc[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+#pragma unroll
+            for (int w = 1; w < D / 16; w <<= 1)
+#pragma unroll
+                for (int ks = 0; ks + w < D / 16; ks += 2 * w) sk[ks][i] += sk[ks + w][i];
+            sacc[i] = sk[0][i];
+        }
+        const bool v0 = g8 < nvalid, v1 = g8 + 8 < nvalid;
+        const float x00 = v0 ? sacc[0] * sl2 : -INFINITY, x01 = v0 ? sacc[1] * sl2 : -INFINITY;
+        const float x10 = v1 ? sacc[2] * sl2 : -INFINITY, x11 = v1 ? sacc[3] * sl2 : -INFINITY;
+        float mx0 = fmaxf(x00, x10), mx1 = fmaxf(x01, x11);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+        }
+        // key 0 of every stage is valid, so the new maxima are finite
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float al0 = mn0 != m0 ? fast_exp2(m0 - mn0) : 1.f;   // 0 when m0 = -inf
+        const float al1 = mn1 != m1 ? fast_exp2(m1 - mn1) : 1.f;
+        m0 = mn0;
+        m1 = mn1;
+        // weights scaled by 2^15 (<= 32768, inside fp16's range): the fp16 head and remainder
+        // below then stay normal numbers down to weights of 2^-17; l and O carry the same
+        // factor, so O / l is unchanged
+        const float r0 = mn0 - DA_P_SHIFT, r1 = mn1 - DA_P_SHIFT;
+        const float p00 = fast_exp2(x00 - r0), p01 = fast_exp2(x01 - r1);
+        const float p10 = fast_exp2(x10 - r0), p11 = fast_exp2(x11 - r1);
+        l0 = l0 * al0 + (p00 + p10);
+        l1 = l1 * al1 + (p01 + p11);
+        // P^T as B: rows = keys, columns = heads.  Each weight is split into an fp16 head and
+        // an fp16 remainder, both multiplied into the same accumulator, so the weights keep ~22
+        // bits: a single fp16 rounding (11 bits) moved the output of a decode step by more
+        // than fp32-vs-fp64 accumulation does.
+        uint32_t ph0 = pack_f16(p00, p01), ph1 = pack_f16(p10, p11);
+        const float2 h0 = __half22float2(*reinterpret_cast<const __half2*>(&ph0));
+        const float2 h1 = __half22float2(*reinterpret_cast<const __half2*>(&ph1));
+        const uint32_t pl0 = pack_f16(p00 - h0.x, p01 - h0.y), pl1 = pack_f16(p10 - h1.x, p11 - h1.y);
+        const uint32_t pb0 = movmatrix_trans(ph0), pb1 = movmatrix_trans(ph1);
+        const uint32_t pr0 = movmatrix_trans(pl0), pr1 = movmatrix_trans(pl1);
+        // O^T: rows = dims 16 m + g8 (+8), columns = heads 2 t4 (+1); this stage's sum in its
+        // own accumulator, folded into the running O with the rescale in fp32
+#pragma unroll
+        for (int m = 0; m < D / 16; ++m) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4_trans(vb + da_off<D>(rv, 2 * m + uv), a0, a1, a2, a3);
+            float so[4] = {0.f, 0.f, 0.f, 0.f};
+            mma16816_f16(so, a0, a1, a2, a3, pb0, pb1);
+            mma16816_f16(so, a0, a1, a2, a3, pr0, pr1);
+            o[m][0] = fmaf(o[m][0], al0, so[0]);
+            o[m][1] = fmaf(o[m][1], al1, so[1]);
+            o[m][2] = fmaf(o[m][2], al0, so[2]);
+            o[m][3] = fmaf(o[m][3], al1, so[3]);
+        }
+        if (st + DA_STAGES < n_st) {
+            // every lane is done with this slot: order its reads before the async-proxy refill
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) issue(st + DA_STAGES);
+            ++issued;
+        }
+    }
+    if (!ok && lane == 0) {
+        // let the loads already issued land before the CTA's shared memory goes away
+        const uint64_t t0 = globaltimer();
+        for (int j = st; j < issued; ++j)
+            while (!mbar_try_wait(wbar + j % DA_STAGES, (uint32_t)(j / DA_STAGES) & 1) &&
+                   globaltimer() - t0 < 1000000ull) {}
+    }
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+    }
     __syncthreads();
-    const int64_t base = (int64_t)blockIdx.x * Hq + g * G;
-    for (int i = threadIdx.x; i < G * D; i += ATT_THREADS) {
+    if (*abort_flag) return;
+    // merge the warps of this CTA (buffers reuse the ring: every load has landed)
+    float* sm_o = reinterpret_cast<float*>(smem);                 // [W][8][D]
+    float* sm_m = sm_o + DA_WARPS * 8 * D;                        // [W][8]
+    float* sm_l = sm_m + DA_WARPS * 8;
+    {
+        float* w0 = sm_o + (warp * 8 + 2 * t4) * D;
+        float* w1 = w0 + D;
+#pragma unroll
+        for (int m = 0; m < D / 16; ++m) {
+            w0[16 * m + g8] = o[m][0];
+            w1[16 * m + g8] = o[m][1];
+            w0[16 * m + g8 + 8] = o[m][2];
+            w1[16 * m + g8 + 8] = o[m][3];
+        }
+        if (g8 == 0) {
+            sm_m[warp * 8 + 2 * t4] = m0; sm_m[warp * 8 + 2 * t4 + 1] = m1;
+            sm_l[warp * 8 + 2 * t4] = l0; sm_l[warp * 8 + 2 * t4 + 1] = l1;
+        }
+    }
+    __syncthreads();
+    const int Hq = Hkv * G;
+    const int64_t base = (int64_t)blockIdx.x * Hq + (int64_t)kvh * G;
+    for (int i = threadIdx.x; i < G * D; i += DA_THREADS) {
         const int h = i / D, d = i % D;
         float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < WARPS; ++w) M = fmaxf(M, sm_m[w][h]);
+        for (int w = 0; w < DA_WARPS; ++w) M = fmaxf(M, sm_m[w * 8 + h]);
         float L = 0.f, O = 0.f;
 #pragma unroll
-        for (int w = 0; w < WARPS; ++w) {
-            const float c = (sm_m[w][h] == -INFINITY) ? 0.f : exp2f(sm_m[w][h] - M);
-            L += c * sm_l[w][h];
-            O += c * sm_o[w][h][d];
+        for (int w = 0; w < DA_WARPS; ++w) {
+            const float mw = sm_m[w * 8 + h];
+            const float c = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+            L += c * sm_l[w * 8 + h];
+            O += c * sm_o[(w * 8 + h) * D + d];
         }
         po[(base + h) * D + d] = O;
         if (d == 0) { pm[base + h] = M; pl[base + h] = L; }
@@ -448,13 +536,17 @@ __global__ void decode_finish_kernel(const int32_t* __restrict__ tok, int32_t* _
     *pos_ptr = pos + 1;
 }
 
-template <int D, int G>
-kvb_status run_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hkv, const int32_t* pos,
-                    int64_t max_pos, int n_blocks, float sl2, float* pm, float* pl, float* po, int* status,
-                    cudaStream_t st) {
+template <int D>
+kvb_status run_attn(const CUtensorMap& tk, const CUtensorMap& tv, const uint16_t* q, int G, int Hkv,
+                    const int32_t* pos, int64_t max_pos, int n_blocks, float sl2, float* pm, float* pl, float* po,
+                    int* status, cudaStream_t st) {
+    static std::atomic<uint64_t> smem_set{0};
+    auto kern = decode_attn_kernel<D>;
+    kvb_status s = ensure_smem_limit((const void*)kern, DaSmem<D>::TOTAL, smem_set, "decode attention smem");
+    if (s != KVB_OK) return s;
     const dim3 grid((unsigned)n_blocks, (unsigned)Hkv);
-    decode_attn_kernel<D, G><<<grid, ATT_THREADS, 0, st>>>(q, kc, vc, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po,
-                                                           status);
+    kern<<<grid, DA_THREADS, DaSmem<D>::TOTAL, st>>>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po,
+                                                     status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode attention launch");
 }
@@ -502,26 +594,28 @@ kvb_status launch_gemv(int mode, const GemvArgs& p, cudaStream_t st) {
 
 // CTA partials of the decode attention for positions below max_pos
 int decode_splits(int64_t max_pos, int) {
-    const int64_t per_block = (int64_t)KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32);
-    return (int)((max_pos + per_block - 1) / per_block);
+    return (int)((max_pos + DA_KEYS_PER_CTA - 1) / DA_KEYS_PER_CTA);
 }
 
 kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hq, int Hkv, int D,
                               const int32_t* pos, int64_t max_pos, float sl2, float* pm, float* pl, float* po,
                               uint16_t* out, int* status, cudaStream_t st) {
+    if (Hkv <= 0 || Hq % Hkv || Hq / Hkv > 8)
+        return fail(KVB_ERR_UNSUPPORTED, "decode attention: at most 8 q heads per kv head (Hq %d, Hkv %d)", Hq, Hkv);
+    if (D != 64 && D != 128) return fail(KVB_ERR_UNSUPPORTED, "decode attention: head_dim %d not built", D);
     const int G = Hq / Hkv;
-    const int n_splits = decode_splits(max_pos, Hkv);
-    kvb_status s;
-#define KVB_DECODE_CASE(DD, GG) \
-    else if (D == DD && G == GG) s = run_attn<DD, GG>(q, kc, vc, Hkv, pos, max_pos, n_splits, sl2, pm, pl, po, status, st);
-    if (false) {}
-    KVB_DECODE_CASE(128, 1) KVB_DECODE_CASE(128, 2) KVB_DECODE_CASE(128, 4) KVB_DECODE_CASE(128, 7) KVB_DECODE_CASE(128, 8)
-    KVB_DECODE_CASE(64, 1) KVB_DECODE_CASE(64, 2) KVB_DECODE_CASE(64, 4) KVB_DECODE_CASE(64, 7) KVB_DECODE_CASE(64, 8)
-#undef KVB_DECODE_CASE
-    else return fail(KVB_ERR_UNSUPPORTED, "decode attention: head_dim %d with %d q heads per kv head not built", D, G);
+    const uint64_t kvd = (uint64_t)Hkv * D;
+    CUtensorMap tk, tv;
+    kvb_status s = make_tmap_2d(&tk, kc, kvd, (uint64_t)max_pos, kvd, 64, DA_STAGE_KEYS);
+    if (s != KVB_OK) return s;
+    s = make_tmap_2d(&tv, vc, kvd, (uint64_t)max_pos, kvd, 64, DA_STAGE_KEYS, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
+    if (s != KVB_OK) return s;
+    const int n_blocks = decode_splits(max_pos, Hkv);
+    s = D == 128 ? run_attn<128>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po, status, st)
+                 : run_attn<64>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po, status, st);
     if (s != KVB_OK) return s;
     decode_combine_kernel<<<dim3((unsigned)Hq, (unsigned)(D / 32)), 32 * COMB_GROUPS, 0, st>>>(
-        pm, pl, po, pos, max_pos, KVB_DECODE_KEYS_PER_SPLIT * (ATT_THREADS / 32), Hq, D, out, status);
+        pm, pl, po, pos, max_pos, DA_KEYS_PER_CTA, Hq, D, out, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode combine launch");
 }

@@ -76,10 +76,14 @@ def test_config_validation_of_rope_scaling_and_groups(kvb):
     bad = kvb.config(synth.YARN_GQA7)
     bad.rs_high = bad.rs_low
     assert L.kvb_workspace_size(C.byref(bad), 100, C.byref(n)) == kvb.KVB_ERR_INVALID_ARG
-    three = kvb.config(synth.LLAMA8B)           # 3 q heads per kv head: prefill yes, decode not built
+    three = kvb.config(synth.LLAMA8B)           # 3 q heads per kv head: prefill and decode
     three.n_q_heads, three.n_kv_heads = 24, 8
     assert L.kvb_workspace_size(C.byref(three), 100, C.byref(n)) == kvb.KVB_OK
-    assert L.kvb_decode_workspace_size(C.byref(three), 100, C.byref(n)) == kvb.KVB_ERR_UNSUPPORTED
+    assert L.kvb_decode_workspace_size(C.byref(three), 100, C.byref(n)) == kvb.KVB_OK
+    wide = kvb.config(synth.LLAMA8B)            # 16 q heads per kv head: prefill yes, decode not built
+    wide.n_q_heads, wide.n_kv_heads = 32, 2
+    assert L.kvb_workspace_size(C.byref(wide), 100, C.byref(n)) == kvb.KVB_OK
+    assert L.kvb_decode_workspace_size(C.byref(wide), 100, C.byref(n)) == kvb.KVB_ERR_UNSUPPORTED
 
 
 def test_workspace_size_grows_with_rows(kvb):

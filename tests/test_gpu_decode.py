@@ -2,6 +2,8 @@
 the split-KV decode attention alone (ragged positions and the 124k headline length),
 and whole decode steps on the tiny and Llama-3.1-8B-shaped 2-layer models, teacher-forced
 on the tokens the GPU produced (the oracle continues from the GPU's prefill cache)."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -36,6 +38,9 @@ def dev(t):
     (L8B, 124160, [124031]),                        # the headline length (124,032 rows)
     (synth.YARN_GQA7, 3000, [0, 1, 1023, 1024, 2999]),   # 7 q heads per kv head, YaRN temperature
     (synth.YARN_GQA7_TINY, 600, [0, 300, 599]),
+    (dataclasses.replace(L8B, n_q_heads=24), 1500, [15, 16, 17, 511, 512, 1499]),   # 3 per kv head
+    (dataclasses.replace(L8B, n_q_heads=32, n_kv_heads=4), 700, [127, 128, 699]),   # 8 per kv head
+    (dataclasses.replace(TINY, n_q_heads=2, n_kv_heads=2), 300, [0, 33, 299]),      # 1 per kv head
 ])
 def test_decode_attention_matches_oracle(kvb, shape, n_rows, positions):
     cfg = kvb.config(shape)
@@ -54,6 +59,31 @@ def test_decode_attention_matches_oracle(kvb, shape, n_rows, positions):
         ref = llama.attention_rows(s, np64(q)[None], np64(k), np64(v), [p])
         e = assert_close_rel(out.cpu().reshape(1, -1), ref.reshape(1, -1), f"decode attention pos {p}", scale=vs)
         print("decode attn", shape.head_dim, n_rows, p, e)
+
+
+def test_decode_attention_ignores_rows_past_the_position(kvb):
+    """Cache rows after `pos` hold NaN (a cache the caller never wrote there): the output is
+    that of the rows up to pos alone."""
+    shape = L8B
+    cfg = kvb.config(shape)
+    n_rows = 700
+    q = synth.randn_bf16((shape.n_q_heads, shape.head_dim), 51)
+    k = synth.randn_bf16((n_rows, shape.n_kv_heads, shape.head_dim), 52)
+    v = synth.randn_bf16((n_rows, shape.n_kv_heads, shape.head_dim), 53).to(torch.float16)
+    ws = kvb.decode_workspace(cfg, n_rows)
+    s = Shape.of(shape)
+    for p in (0, 9, 130, 511, 600):
+        kn, vn = k.clone(), v.clone()
+        kn[p + 1:] = float("nan")
+        vn[p + 1:] = float("nan")
+        out = kvb.decode_attention(cfg, dev(q), dev(kn), dev(vn), torch.tensor([p], dtype=torch.int32, device="cuda"),
+                                   n_rows, ws=ws)
+        torch.cuda.synchronize()
+        assert kvb.device_status(ws) == 0
+        assert torch.isfinite(out.float()).all(), p
+        ref = llama.attention_rows(s, np64(q)[None], np64(k), np64(v), [p])
+        assert_close_rel(out.cpu().reshape(1, -1), ref.reshape(1, -1), f"decode attention pos {p} (NaN after)",
+                         scale=float(np.sqrt(np.mean(np64(v) ** 2))))
 
 
 def test_decode_attention_rejects_position_out_of_range(kvb):
