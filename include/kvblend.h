@@ -429,8 +429,10 @@ kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const 
 /* The decode step's attention alone: the new row's q (bf16 [Hq][D], RoPE applied)
  * over one layer's cache rows [0, *pos] (k_layer bf16, v_layer fp16 holding
  * bf16-precision values, both [n_rows][Hkv][D], n_rows >= max_pos); causal softmax
- * with scale 1/sqrt(D), GQA head map q head h -> kv head h / (Hq/Hkv).
- * out: bf16 [Hq][D].  Split-KV over 128-row splits, merged by log-sum-exp.
+ * with the config's scale (kvb_attention_scale), GQA head map q head h -> kv head
+ * h / (Hq/Hkv), at most 8 q heads per kv head.
+ * out: bf16 [Hq][D].  Split-KV (one split per warp, all splits resident at once), merged
+ * by log-sum-exp.
  * Workspace and errors as kvb_decode_step. */
 kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const uint16_t* k_layer,
                                 const uint16_t* v_layer, int64_t n_rows, const int32_t* pos, int64_t max_pos,

@@ -5,8 +5,8 @@
 // kernels are CUDA-core kernels built for streaming, not tensor-core tiles:
 //   decode_embed      - x = embed[tokens[pos]] (fp32)
 //   gemv_kernel       - y = W a for one activation row held in shared memory as bf16;
-//                       warp per output row (or row pair), 16-byte weight loads, 8-16 per
-//                       lane in flight.  QKV and SwiGLU normalise the residual row
+//                       warp per output row (or row pair), 16-byte weight loads, 8 per
+//                       lane in flight, all warps resident at once.  QKV and SwiGLU normalise the residual row
 //                       themselves (RMSNorm prologue in every block); QKV computes the two
 //                       rows of a rotation pair in one warp, applies RoPE at `pos` and writes
 //                       q and the cache's K/V row `pos` (V as bf16-rounded fp16, like the
@@ -112,8 +112,10 @@ KVB_DEV void dot_rows(const uint16_t* __restrict__ w1, const uint16_t* __restric
 //                 `pos`, bf16 q or cache K row `pos`; or one V row (+ bias): cache V row `pos`
 //   GEMV_RESID  - one row: x[n] += y
 //   GEMV_SWIGLU - gate row n and up row n: h[n] = bf16(silu(gate) * up)
+// Four blocks per SM (<= 64 registers a thread): 32 warps per SM hold every row of the
+// 4096-row GEMVs at once, so no warp takes a second row while others idle.
 template <int MODE>
-__global__ void __launch_bounds__(GEMV_THREADS)
+__global__ void __launch_bounds__(GEMV_THREADS, 4)
 gemv_kernel(const GemvArgs p) {
     extern __shared__ __align__(16) uint16_t act[];   // [K]
     __shared__ float red[GEMV_THREADS / 32];
@@ -158,7 +160,7 @@ gemv_kernel(const GemvArgs p) {
             if (u < n_pairs) {
                 const int h = (int)(u / half), i = (int)(u % half);
                 float a, b;
-                dot_rows<true, 8>(p.W + ((int64_t)h * D + i) * K, p.W + ((int64_t)h * D + i + half) * K, act, K, lane,
+                dot_rows<true, 4>(p.W + ((int64_t)h * D + i) * K, p.W + ((int64_t)h * D + i + half) * K, act, K, lane,
                                   a, b);
                 if (lane == 0) {
                     if (p.bias) {
@@ -175,7 +177,7 @@ gemv_kernel(const GemvArgs p) {
             } else {
                 const int j = (int)(u - n_pairs);
                 float a, unused;
-                dot_rows<false, 16>(p.W + ((int64_t)(Hq + Hkv) * D + j) * K, nullptr, act, K, lane, a, unused);
+                dot_rows<false, 8>(p.W + ((int64_t)(Hq + Hkv) * D + j) * K, nullptr, act, K, lane, a, unused);
                 if (lane == 0) {
                     if (p.bias) a += p.bias[(int64_t)(Hq + Hkv) * D + j];
                     const float v = __bfloat162float(__float2bfloat16_rn(a));
@@ -187,10 +189,10 @@ gemv_kernel(const GemvArgs p) {
         for (int64_t n = first; n < p.N; n += warps) {
             float a, b;
             if constexpr (MODE == GEMV_SWIGLU) {
-                dot_rows<true, 8>(p.W + n * K, p.W2 + n * K, act, K, lane, a, b);
+                dot_rows<true, 4>(p.W + n * K, p.W2 + n * K, act, K, lane, a, b);
                 if (lane == 0) p.y_bf16[n] = __bfloat16_as_ushort(__float2bfloat16_rn(a / (1.0f + __expf(-a)) * b));
             } else {
-                dot_rows<false, 16>(p.W + n * K, nullptr, act, K, lane, a, b);
+                dot_rows<false, 8>(p.W + n * K, nullptr, act, K, lane, a, b);
                 if (lane == 0) p.y_f32[n] += a;
             }
         }
@@ -199,10 +201,11 @@ gemv_kernel(const GemvArgs p) {
 
 // ---------------------------------------------------------------- decode attention
 //
-// One CTA = DA_WARPS warps of one kv head; warp w takes the split of
-// KVB_DECODE_KEYS_PER_SPLIT cache rows starting at (blockIdx.x * DA_WARPS + w) * split and
-// streams it through its own ring of DA_STAGES stages of 16 rows (K and V tiles loaded by
-// TMA, 128-byte swizzle).  Per stage, with the G <= 8 q heads of the group as the 8
+// One CTA = DA_WARPS warps of one kv head; warp w takes the split of `split` cache rows
+// starting at (blockIdx.x * DA_WARPS + w) * split and streams it through its own ring of
+// DA_STAGES stages of 16 rows (K and V tiles loaded by TMA, 128-byte swizzle).  The host
+// sizes the splits so that all CTAs are resident at once (one wave: two CTAs per SM), so
+// every warp pays the pipeline start-up once.  Per stage, with the G <= 8 q heads of the group as the 8
 // columns of mma.sync m16n8k16 tiles (columns G..7 are zero q heads, never written out):
 //   S^T [16 keys x 8 heads] = K [16 x D] . Q^T            (bf16, fp32 accumulate)
 //   online softmax per head (column) in the log2 domain;
@@ -217,7 +220,8 @@ constexpr int DA_WARPS = 4;
 constexpr int DA_THREADS = 32 * DA_WARPS;
 constexpr int DA_STAGE_KEYS = 16;
 constexpr int DA_STAGES = 3;
-constexpr int DA_KEYS_PER_CTA = KVB_DECODE_KEYS_PER_SPLIT * DA_WARPS;
+constexpr int DA_CTAS_PER_SM = 2;
+constexpr int DA_MAX_SLOTS = 384;            // bound on resident CTAs (2 per SM, up to 192 SMs)
 constexpr float DA_P_SHIFT = 15.f;           // softmax weights carried as p * 2^15
 
 template <int D>
@@ -277,8 +281,8 @@ template <int D>
 __global__ void __launch_bounds__(DA_THREADS, 2)
 decode_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const uint16_t* __restrict__ q, int G, int Hkv, const int32_t* __restrict__ pos_ptr,
-                   int64_t max_pos, int n_blocks, float sl2, float* __restrict__ pm, float* __restrict__ pl,
-                   float* __restrict__ po, int* status) {
+                   int64_t max_pos, int n_blocks, int split, float sl2, float* __restrict__ pm,
+                   float* __restrict__ pl, float* __restrict__ po, int* status) {
     using S = DaSmem<D>;
     constexpr int NB = S::NB;
     extern __shared__ uint8_t smem_raw[];
@@ -299,8 +303,8 @@ decode_attn_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constan
     if (threadIdx.x == 32) { prefetch_tmap(&tmK); prefetch_tmap(&tmV); }
     __syncthreads();
 
-    const int64_t start = ((int64_t)blockIdx.x * DA_WARPS + warp) * KVB_DECODE_KEYS_PER_SPLIT;
-    int64_t end = start + KVB_DECODE_KEYS_PER_SPLIT;
+    const int64_t start = ((int64_t)blockIdx.x * DA_WARPS + warp) * split;
+    int64_t end = start + split;
     if (end > (int64_t)pos + 1) end = (int64_t)pos + 1;
     const int n_st = start < end ? (int)((end - start + DA_STAGE_KEYS - 1) / DA_STAGE_KEYS) : 0;
     uint8_t* ring = smem + warp * DA_STAGES * S::STAGE;
@@ -538,15 +542,15 @@ __global__ void decode_finish_kernel(const int32_t* __restrict__ tok, int32_t* _
 
 template <int D>
 kvb_status run_attn(const CUtensorMap& tk, const CUtensorMap& tv, const uint16_t* q, int G, int Hkv,
-                    const int32_t* pos, int64_t max_pos, int n_blocks, float sl2, float* pm, float* pl, float* po,
-                    int* status, cudaStream_t st) {
+                    const int32_t* pos, int64_t max_pos, int n_blocks, int split, float sl2, float* pm, float* pl,
+                    float* po, int* status, cudaStream_t st) {
     static std::atomic<uint64_t> smem_set{0};
     auto kern = decode_attn_kernel<D>;
     kvb_status s = ensure_smem_limit((const void*)kern, DaSmem<D>::TOTAL, smem_set, "decode attention smem");
     if (s != KVB_OK) return s;
     const dim3 grid((unsigned)n_blocks, (unsigned)Hkv);
-    kern<<<grid, DA_THREADS, DaSmem<D>::TOTAL, st>>>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po,
-                                                     status);
+    kern<<<grid, DA_THREADS, DaSmem<D>::TOTAL, st>>>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, split, sl2, pm, pl,
+                                                     po, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode attention launch");
 }
@@ -592,9 +596,12 @@ kvb_status launch_gemv(int mode, const GemvArgs& p, cudaStream_t st) {
     }
 }
 
-// CTA partials of the decode attention for positions below max_pos
-int decode_splits(int64_t max_pos, int) {
-    return (int)((max_pos + DA_KEYS_PER_CTA - 1) / DA_KEYS_PER_CTA);
+// Bound on the CTA partials (per kv head) of the decode attention for positions below
+// max_pos: the workspace is laid out with it, whatever device runs the kernel.
+int decode_splits(int64_t max_pos, int Hkv) {
+    const int64_t by_rows = (max_pos + DA_WARPS * DA_STAGE_KEYS - 1) / (DA_WARPS * DA_STAGE_KEYS);
+    const int64_t by_slots = Hkv > 0 && DA_MAX_SLOTS / Hkv > 0 ? DA_MAX_SLOTS / Hkv : 1;
+    return (int)(by_rows < by_slots ? by_rows : by_slots);
 }
 
 kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, int Hq, int Hkv, int D,
@@ -610,12 +617,21 @@ kvb_status launch_decode_attn(const uint16_t* q, const uint16_t* kc, const uint1
     if (s != KVB_OK) return s;
     s = make_tmap_2d(&tv, vc, kvd, (uint64_t)max_pos, kvd, 64, DA_STAGE_KEYS, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
     if (s != KVB_OK) return s;
-    const int n_blocks = decode_splits(max_pos, Hkv);
-    s = D == 128 ? run_attn<128>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po, status, st)
-                 : run_attn<64>(tk, tv, q, G, Hkv, pos, max_pos, n_blocks, sl2, pm, pl, po, status, st);
+    // one wave: at most DA_CTAS_PER_SM CTAs per SM over all kv heads, each warp's split a
+    // multiple of the 16-row stage, the splits covering rows [0, max_pos)
+    int64_t n_blocks = (int64_t)DA_CTAS_PER_SM * num_sms() / Hkv;
+    const int cap = decode_splits(max_pos, Hkv);
+    if (n_blocks > cap) n_blocks = cap;
+    if (n_blocks < 1) n_blocks = 1;
+    int64_t split = (max_pos + n_blocks * DA_WARPS - 1) / (n_blocks * DA_WARPS);
+    split = (split + DA_STAGE_KEYS - 1) / DA_STAGE_KEYS * DA_STAGE_KEYS;
+    n_blocks = (max_pos + split * DA_WARPS - 1) / (split * DA_WARPS);
+    if (split > 0x7FFFFFFF / DA_WARPS) return fail(KVB_ERR_INVALID_ARG, "decode attention: max_pos too large");
+    s = D == 128 ? run_attn<128>(tk, tv, q, G, Hkv, pos, max_pos, (int)n_blocks, (int)split, sl2, pm, pl, po, status, st)
+                 : run_attn<64>(tk, tv, q, G, Hkv, pos, max_pos, (int)n_blocks, (int)split, sl2, pm, pl, po, status, st);
     if (s != KVB_OK) return s;
     decode_combine_kernel<<<dim3((unsigned)Hq, (unsigned)(D / 32)), 32 * COMB_GROUPS, 0, st>>>(
-        pm, pl, po, pos, max_pos, DA_KEYS_PER_CTA, Hq, D, out, status);
+        pm, pl, po, pos, max_pos, (int)(split * DA_WARPS), Hq, D, out, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "decode combine launch");
 }

@@ -111,7 +111,6 @@ kvb_status launch_deviation_histogram(const uint16_t* ka, int64_t lda, const uin
                                       int kv_dim, const float* edges, int n_edges, float* dev,
                                       unsigned long long* hist, cudaStream_t st);
 // ---------------------------------------------------------------- greedy decode
-constexpr int KVB_DECODE_KEYS_PER_SPLIT = 128;   // cache rows per warp split of the decode attention
 constexpr int KVB_DECODE_MAX_K = 16384;          // longest input row of a decode GEMV (shared memory)
 enum GemvMode { GEMV_QKV = 0, GEMV_RESID = 1, GEMV_SWIGLU = 2 };
 struct GemvArgs {

@@ -10,7 +10,8 @@
 Shapes are the Llama-3.1-8B layer (H 4096, 32 q / 8 kv heads, D 128, F 14336).  The
 selected rows of `attn` are drawn uniformly over the context (as the HKVD choice of
 r = m / n_kv would spread them) and always include the last row.  Prints the CUDA-event
-time of the last repetition and its algorithmic throughput.
+time of the last repetition (the mean of the last --timed calls) and its algorithmic
+throughput.
 """
 from __future__ import annotations
 
@@ -32,6 +33,9 @@ def main():
     ap.add_argument("--layers", type=int, default=2)
     ap.add_argument("--which", default="qkv", choices=["qkv", "o", "gateup", "down"])
     ap.add_argument("--reps", type=int, default=2)
+    ap.add_argument("--timed", type=int, default=1,
+                    help="calls between the timing events (the mean is reported); more than one keeps the "
+                         "host's launch overhead out of short kernels' times")
     a = ap.parse_args()
     build.build()
     shape = synth.LLAMA8B
@@ -124,10 +128,11 @@ def main():
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    fn()
+    for _ in range(max(a.timed, 1)):
+        fn()
     e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    ms = e0.elapsed_time(e1) / max(a.timed, 1)
     assert kvb.device_status(ws) == 0
     out.update(kernel=a.kernel, ms=round(ms, 4))
     if flop:
