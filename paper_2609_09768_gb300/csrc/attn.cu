@@ -11,7 +11,8 @@
 // Both A operands live in tensor memory, so each MMA reads only its K or V tile
 // from shared memory: with A and B both in shared memory an M128 x N128 step
 // needs the whole shared-memory bandwidth on its own, before the TMA writes.
-// TMEM columns: S double buffer [0, 256), O [256, 384), Q [384, 448), P [448, 512).
+// TMEM columns: S double buffer [0, 256) (P_j is written over the first half of S_j's
+// buffer), O [256, 384), Q [384, 448).
 //
 // Pipeline per key tile j (128 keys):
 //   TMA warp   : K_j and V_j together into a 3-deep ring (128-byte swizzle); slot
@@ -22,7 +23,10 @@
 //   4 softmax warps (thread = row): load the row's Q into TMEM once; per tile
 //                read S_j from TMEM, mask, online softmax with a lazily updated
 //                running max (O is rescaled only when the max grows by more than
-//                2^8), write P_j into its TMEM columns once P.V_{j-1} is done.
+//                2^8, after P.V_{j-1} is done), write P_j over S_j.  The buffer's
+//                previous P (tile j-2) was read by P.V_{j-2}, which ran before S_j
+//                (MMAs complete in issue order), so the common path waits for
+//                nothing but S_j.
 // Lazy rescaling keeps the result exact: every term uses the same reference max
 // as the running sum it is divided by.
 // Precision: Q.K^T runs on bf16 operands; P.V runs on fp16 operands - the
@@ -41,7 +45,7 @@ constexpr int THREADS = 192;
 constexpr int KT_ROWS = 128;                 // keys per tile
 constexpr int STAGES = 3;                    // K and V ring depth
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t COL_S = 0, COL_O = 256, COL_Q = 384, COL_P = 448;
+constexpr uint32_t COL_S = 0, COL_O = 256, COL_Q = 384;
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
 
@@ -67,7 +71,8 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     // hundreds of cycles, so each 128-key tile uses two of each: kv_full (K_j and V_j
     // landed) and p_full (P_{j-1} written) for the MMA thread; s_full (S_j done) and
     // pv_done (P.V_i done) as commits.  P.V_i done also frees slot i % STAGES for the
-    // producer (P_i was written after S_i had been read) and lets the softmax overwrite P.
+    // producer (P_i was written after S_i had been read) and tells a softmax that must
+    // rescale O that the accumulation it rescales is complete.
     uint64_t* q_ready = bars + 0;                // Q rows stored into TMEM (4 warps)
     uint64_t* kv_full = bars + 1;                // [STAGES]: K_j and V_j in slot j % STAGES
     uint64_t* s_full = kv_full + STAGES;         // [2]: S_j done, phase j/2 of s_full[j % 2]
@@ -187,7 +192,8 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     if (!mbar_wait(&p_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
                     tc_fence_after();
                     const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
-                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_P;
+                    // P_i sits in the first half of its own S buffer
+                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * KT_ROWS;
                     mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
 #pragma unroll
                     for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
@@ -277,14 +283,17 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             }
             l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
 
-            if (j >= 1) {
+            // O is rescaled only once P.V_{j-1} has finished accumulating into it; P_j itself
+            // goes into S buffer b, whose previous P (of tile j-2) was read by P.V_{j-2}
+            // before S_j was written (the MMAs run in issue order)
+            if (j >= 1 && __any_sync(0xffffffffu, resc)) {
                 if (!mbar_wait_warp(&pv_done[(j - 1) % STAGES], (uint32_t)((j - 1) / STAGES) & 1, abort_flag,
                                     p.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, resc)) {
+                {
                     const uint32_t oaddr = tmem_base + lane_addr + COL_O;
 #pragma unroll 1
                     for (int c = 0; c < D / 32; ++c) {
@@ -298,9 +307,9 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     tmem_st_wait();
                 }
             }
-            // P row L (fp16 pairs) into its TMEM columns; P.V_{j-1} has finished reading them
-            tmem_st32(tmem_base + lane_addr + COL_P, pk);
-            tmem_st32(tmem_base + lane_addr + COL_P + 32, pk + 32);
+            // P row L (fp16 pairs) over the S_j it was computed from
+            tmem_st32(tmem_base + lane_addr + COL_S + b * KT_ROWS, pk);
+            tmem_st32(tmem_base + lane_addr + COL_S + b * KT_ROWS + 32, pk + 32);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
