@@ -3,21 +3,25 @@
 // Each CTA owns one (block of query rows, kv head) unit.  The G = Hq/Hkv query heads
 // that share kv head g are packed with RPB = floor(128/G) query rows into the 128
 // rows of one MMA tile (lane = row_in_block * G + head_in_group; the last 128 - RPB*G
-// lanes idle when G does not divide 128), so every K/V tile loaded serves all G heads.  Row r attends cache rows [lo_r, hi_r] where hi_r is
-// the row's own cache index: this one predicate covers the sparse recompute rows
-// of the selective layers, the dense causal prefill and the block-diagonal
-// per-chunk prefill.
+// lanes idle when G does not divide 128), so every K/V tile loaded serves all G heads.
+// Row r attends cache rows [lo_r, hi_r] where hi_r is the row's own cache index: this
+// one predicate covers the sparse recompute rows of the selective layers, the dense
+// causal prefill and the block-diagonal per-chunk prefill.
 //
 // Both A operands live in tensor memory, so each MMA reads only its K or V tile
 // from shared memory: with A and B both in shared memory an M128 x N128 step
 // needs the whole shared-memory bandwidth on its own, before the TMA writes.
-// TMEM columns: S double buffer [0, 256) (P_j is written over the first half of S_j's
-// buffer), O [256, 384), Q [384, 448).
+// Key tiles are 144 rows: the widest that leaves room in the 512 TMEM columns for two S
+// buffers, O and Q while three K/V stages (216 KB) fit in shared memory; every tile's
+// barrier waits and commits on the issuing thread then cover 1,152 cycles of MMAs
+// instead of 1,024 with 128-key tiles.
+// TMEM columns: S buffers [0, 144) and [160, 304) (P_j is written over the first 72
+// columns of S_j's buffer), O [320, 448), Q [448, 512).
 //
-// Pipeline per key tile j (128 keys):
+// Pipeline per key tile j (144 keys):
 //   TMA warp   : K_j and V_j together into a 3-deep ring (128-byte swizzle); slot
 //                j % 3 is reused once P.V of the tile that held it has completed
-//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=128, K=16 steps,
+//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=144, K=16 steps,
 //                A = Q from TMEM); after the softmax of tile j-1,
 //                O += P_{j-1} V_{j-1} (A = P from TMEM, V an MN-major operand)
 //   4 softmax warps (thread = row): load the row's Q into TMEM once; per tile
@@ -42,16 +46,16 @@ namespace kvb {
 namespace {
 
 constexpr int THREADS = 192;
-constexpr int KT_ROWS = 128;                 // keys per tile
+constexpr int KT_ROWS = 144;                 // keys per tile
 constexpr int STAGES = 3;                    // K and V ring depth
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t COL_S = 0, COL_O = 256, COL_Q = 384;
+constexpr uint32_t COL_S = 0, S_STRIDE = 160, COL_O = 320, COL_Q = 448;   // S buffers 32-column aligned
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
 
 template <int D>
 struct Smem {
-    static constexpr int CHUNK = 128 * 128;              // 128 rows x 128 bytes
+    static constexpr int CHUNK = KT_ROWS * 128;          // KT_ROWS rows x 128 bytes
     static constexpr int KV_BYTES = (D / 64) * CHUNK;    // one K or V tile
     static constexpr int OFF_K = 0;
     static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
@@ -68,7 +72,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     // Every wait of the MMA thread and every tcgen05.commit costs the tensor pipe tens to
-    // hundreds of cycles, so each 128-key tile uses two of each: kv_full (K_j and V_j
+    // hundreds of cycles, so each key tile uses two of each: kv_full (K_j and V_j
     // landed) and p_full (P_{j-1} written) for the MMA thread; s_full (S_j done) and
     // pv_done (P.V_i done) as commits.  P.V_i done also frees slot i % STAGES for the
     // producer (P_i was written after S_i had been read) and tells a softmax that must
@@ -177,7 +181,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     // descriptor built once per tile; constant steps inside the unrolled loop keep
                     // the issuing thread ahead of the 64-cycle MMAs
                     const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
-                    const uint32_t sd = tmem_base + COL_S + b * KT_ROWS, qa = tmem_base + COL_Q;
+                    const uint32_t sd = tmem_base + COL_S + b * S_STRIDE, qa = tmem_base + COL_Q;
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
                         // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
@@ -193,7 +197,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     tc_fence_after();
                     const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
                     // P_i sits in the first half of its own S buffer
-                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * KT_ROWS;
+                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * S_STRIDE;
                     mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
 #pragma unroll
                     for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
@@ -240,7 +244,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             tc_fence_after();
             uint32_t s[KT_ROWS];
 #pragma unroll
-            for (int c = 0; c < KT_ROWS / 32; ++c) tmem_ld32(tmem_base + lane_addr + b * KT_ROWS + c * 32, s + c * 32);
+            for (int c = 0; c < KT_ROWS / 32; ++c) tmem_ld32(tmem_base + lane_addr + b * S_STRIDE + c * 32, s + c * 32);
+            if constexpr (KT_ROWS % 32)
+                tmem_ld16(tmem_base + lane_addr + b * S_STRIDE + (KT_ROWS / 32) * 32,
+                          *reinterpret_cast<uint32_t(*)[16]>(s + (KT_ROWS / 32) * 32));
             tmem_ld_wait();
 
             const int key0 = (t_begin + j) * KT_ROWS;
@@ -308,8 +315,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                 }
             }
             // P row L (fp16 pairs) over the S_j it was computed from
-            tmem_st32(tmem_base + lane_addr + COL_S + b * KT_ROWS, pk);
-            tmem_st32(tmem_base + lane_addr + COL_S + b * KT_ROWS + 32, pk + 32);
+            tmem_st32(tmem_base + lane_addr + COL_S + b * S_STRIDE, pk);
+            tmem_st32(tmem_base + lane_addr + COL_S + b * S_STRIDE + 32, pk + 32);
+            static_assert(KT_ROWS == 144, "P store covers 72 columns");
+            tmem_st8(tmem_base + lane_addr + COL_S + b * S_STRIDE + 64, pk + 64);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
