@@ -259,12 +259,17 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                     if (key > hi || key < lo) s[c] = __float_as_uint(-INFINITY);
                 }
             }
-            // row max as a tree: 16 independent chains, not one 128-long dependent chain
+            // row max as a tree: 16 independent chains of three-input maxima, not one
+            // 144-long dependent chain
+            static_assert((KT_ROWS - 16) % 32 == 0, "max tree takes 32 keys per step");
             float mx[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c) mx[c] = __uint_as_float(s[c]);
 #pragma unroll
-            for (int c = 16; c < KT_ROWS; ++c) mx[c & 15] = fmaxf(mx[c & 15], __uint_as_float(s[c]));
+            for (int c = 16; c < KT_ROWS; c += 32)
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                    mx[e] = fmax3(mx[e], __uint_as_float(s[c + e]), __uint_as_float(s[c + 16 + e]));
 #pragma unroll
             for (int w = 8; w > 0; w >>= 1)
 #pragma unroll
@@ -279,16 +284,23 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                 m_run = m_new;
             }
             const float mref = ((m_run == -INFINITY) ? 0.f : m_run * sl2) - P_SHIFT_LOG2;
+            // exponents and row sums on key pairs: one FFMA2 and one FADD2 per two keys
             uint32_t pk[KT_ROWS / 2];
-            float ls[4] = {0.f, 0.f, 0.f, 0.f};
+            const uint64_t sl2x2 = f2_pack(sl2, sl2), nmref2 = f2_pack(-mref, -mref);
+            uint64_t ls2[4] = {0ull, 0ull, 0ull, 0ull};   // (even keys, odd keys) partial sums
 #pragma unroll
             for (int c = 0; c < KT_ROWS; c += 2) {
-                const float e0 = fast_exp2(fmaf(__uint_as_float(s[c]), sl2, -mref));
-                const float e1 = fast_exp2(fmaf(__uint_as_float(s[c + 1]), sl2, -mref));
-                ls[(c >> 1) & 3] += e0 + e1;
+                float a0, a1;
+                f2_unpack(f2_fma(f2_pack(__uint_as_float(s[c]), __uint_as_float(s[c + 1])), sl2x2, nmref2), a0, a1);
+                const float e0 = fast_exp2(a0), e1 = fast_exp2(a1);
+                ls2[(c >> 1) & 3] = f2_add(ls2[(c >> 1) & 3], f2_pack(e0, e1));
                 pk[c / 2] = pack_f16(e0, e1);
             }
-            l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+            {
+                float l_even, l_odd;
+                f2_unpack(f2_add(f2_add(ls2[0], ls2[1]), f2_add(ls2[2], ls2[3])), l_even, l_odd);
+                l_run += l_even + l_odd;
+            }
 
             // O is rescaled only once P.V_{j-1} has finished accumulating into it; P_j itself
             // goes into S buffer b, whose previous P (of tile j-2) was read by P.V_{j-2}

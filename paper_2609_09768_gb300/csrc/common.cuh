@@ -252,6 +252,31 @@ KVB_DEV float fast_exp2(float x) {
     return y;
 }
 
+// Paired fp32 arithmetic (sm_100-family FFMA2/FADD2: one instruction for two lanes of
+// a 64-bit register pair, each lane rounded exactly like the scalar instruction) and
+// the three-input max; the attention softmax uses them to halve its issue count.
+KVB_DEV uint64_t f2_pack(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+KVB_DEV void f2_unpack(uint64_t v, float& lo, float& hi) { asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v)); }
+KVB_DEV uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+KVB_DEV uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+KVB_DEV float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 KVB_DEV uint32_t warp_id() { return threadIdx.x >> 5; }
 KVB_DEV uint32_t lane_id() { return threadIdx.x & 31; }
 
