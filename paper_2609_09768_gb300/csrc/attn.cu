@@ -22,7 +22,8 @@
 //   TMA warp   : K_j and V_j together into a 3-deep ring (128-byte swizzle); slot
 //                j % 3 is reused once P.V of the tile that held it has completed
 //   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=144, K=16 steps,
-//                A = Q from TMEM); after the softmax of tile j-1,
+//                A = Q from TMEM); after the softmax of tile j-1 (a named barrier that
+//                the softmax warps arrive on and the MMA warp blocks on),
 //                O += P_{j-1} V_{j-1} (A = P from TMEM, V an MN-major operand)
 //   4 softmax warps (thread = row): load the row's Q into TMEM once; per tile
 //                read S_j from TMEM, mask, online softmax with a lazily updated
@@ -50,6 +51,12 @@ constexpr int KT_ROWS = 144;                 // keys per tile
 constexpr int STAGES = 3;                    // K and V ring depth
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t COL_S = 0, S_STRIDE = 160, COL_O = 320, COL_Q = 448;   // S buffers 32-column aligned
+// P_j written -> MMA warp: one named barrier that the 4 softmax warps and the MMA warp
+// all pass with bar.sync once per key tile, in lockstep, on every path (also after a
+// failed wait), so each phase completes and no warp can arrive twice in one phase.  The
+// softmax warps lose nothing by blocking there: the S MMA they wait for next was issued
+// before the MMA warp reached the barrier.
+constexpr uint32_t BAR_P = 1, BAR_P_COUNT = 5 * 32;
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
 
@@ -73,15 +80,15 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     // Every wait of the MMA thread and every tcgen05.commit costs the tensor pipe tens to
     // hundreds of cycles, so each key tile uses two of each: kv_full (K_j and V_j
-    // landed) and p_full (P_{j-1} written) for the MMA thread; s_full (S_j done) and
-    // pv_done (P.V_i done) as commits.  P.V_i done also frees slot i % STAGES for the
-    // producer (P_i was written after S_i had been read) and tells a softmax that must
-    // rescale O that the accumulation it rescales is complete.
+    // landed, an mbarrier) and P_{j-1} written (the named barrier BAR_P) for the MMA
+    // warp; s_full (S_j done) and pv_done (P.V_i done) as commits.  P.V_i done also
+    // frees slot i % STAGES for the producer (P_i was written after S_i had been read)
+    // and tells a softmax that must rescale O that the accumulation it rescales is
+    // complete.
     uint64_t* q_ready = bars + 0;                // Q rows stored into TMEM (4 warps)
     uint64_t* kv_full = bars + 1;                // [STAGES]: K_j and V_j in slot j % STAGES
     uint64_t* s_full = kv_full + STAGES;         // [2]: S_j done, phase j/2 of s_full[j % 2]
-    uint64_t* p_full = s_full + 2;               // [STAGES]: P_j written, phase j/3 of p_full[j % 3]
-    uint64_t* pv_done = p_full + STAGES;         // [STAGES]: P.V_i done, phase i/3 of pv_done[i % 3]
+    uint64_t* pv_done = s_full + 2;              // [STAGES]: P.V_i done, phase i/3 of pv_done[i % 3]
     uint64_t* drain = pv_done + STAGES;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -98,7 +105,6 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
         mbar_init(q_ready, 4);
         for (int st = 0; st < STAGES; ++st) {
             mbar_init(&kv_full[st], 1);
-            mbar_init(&p_full[st], 4);
             mbar_init(&pv_done[st], 1);
         }
         for (int b = 0; b < 2; ++b) mbar_init(&s_full[b], 1);
@@ -164,52 +170,64 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             }
         }
     } else if (warp == 1) {
-        if (lane == 0 && n_tiles > 0) {
-            // ------------------------------------------------ MMA issuer
+        if (n_tiles > 0) {
+            // ------------------------------------------------ MMA issuer (lane 0; the whole warp
+            // takes part in the named-barrier waits for P)
             constexpr uint32_t IDESC_S = idesc_bf16(128, KT_ROWS, false);
             constexpr uint32_t IDESC_O = idesc_f16kind(128, D, true, false);   // fp16 P and V
             const uint32_t k0 = smem_u32(sK), v0 = smem_u32(sV);
-            bool ok = mbar_wait(q_ready, 0, abort_flag, p.status);
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(q_ready, 0, abort_flag, p.status);
             tc_fence_after();
-            for (int j = 0; ok && j <= n_tiles; ++j) {
-                if (j < n_tiles) {
+            for (int j = 0; j <= n_tiles; ++j) {
+                if (j < n_tiles && lane == 0 && ok) {
                     const int b = j & 1, st = j % STAGES;
                     // S buffer b last held S_{j-2}: the softmax read it before writing P_{j-2},
-                    // which this thread waited for in the previous iteration
-                    if (!mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status)) break;
-                    tc_fence_after();
-                    // descriptor built once per tile; constant steps inside the unrolled loop keep
-                    // the issuing thread ahead of the 64-cycle MMAs
-                    const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
-                    const uint32_t sd = tmem_base + COL_S + b * S_STRIDE, qa = tmem_base + COL_Q;
+                    // which P.V_{j-2} (issued before this MMA, so executed before it) consumed
+                    ok = mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status);
+                    if (ok) {
+                        tc_fence_after();
+                        // descriptor built once per tile; constant steps inside the unrolled loop keep
+                        // the issuing thread ahead of the MMAs
+                        const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
+                        const uint32_t sd = tmem_base + COL_S + b * S_STRIDE, qa = tmem_base + COL_Q;
 #pragma unroll
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
-                        mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32), IDESC_S,
-                                   kk > 0 ? 1u : 0u);
+                        for (int kk = 0; kk < D / 16; ++kk) {
+                            // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
+                            mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32),
+                                       IDESC_S, kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(&s_full[b]);
                     }
-                    mma_commit(&s_full[b]);
                 }
                 if (j >= 1) {
                     const int i = j - 1, st = i % STAGES;
-                    // V_i landed with K_i (kv_full waited in iteration i)
-                    if (!mbar_wait(&p_full[st], (uint32_t)(i / STAGES) & 1, abort_flag, p.status)) break;
-                    tc_fence_after();
-                    const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
-                    // P_i sits in the first half of its own S buffer
-                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * S_STRIDE;
-                    mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
+                    // P_i written by all four softmax warps: a blocking hardware barrier, not a
+                    // polling loop, so the issuing thread takes no data-dependent branch here
+                    __syncwarp();
+                    named_bar_sync(BAR_P, BAR_P_COUNT);
+                    if (lane == 0 && ok) {
+                        tc_fence_after();
+                        // V_i landed with K_i (kv_full waited in iteration i)
+                        const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
+                        // P_i sits in the first half of its own S buffer
+                        const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * S_STRIDE;
+                        mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
 #pragma unroll
-                    for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
-                        // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
-                        mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
+                        for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
+                            // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
+                            mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
+                        }
+                        mma_commit(&pv_done[st]);
                     }
-                    mma_commit(&pv_done[st]);
                 }
             }
-            mma_commit(drain);
-            const uint64_t t0 = globaltimer();
-            while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            if (lane == 0) {
+                mma_commit(drain);
+                const uint64_t t0 = globaltimer();
+                while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+            }
+            __syncwarp();
         }
     } else if (n_tiles > 0) {
         // ---------------------------------------------------- softmax warps (2..5)
@@ -240,7 +258,13 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
         }
         for (int j = 0; j < n_tiles; ++j) {
             const int b = j & 1;
-            if (!mbar_wait_warp(&s_full[b], (j >> 1) & 1, abort_flag, p.status)) { ok = false; break; }
+            // after a failed wait the warp keeps looping without work, so that it still
+            // passes every tile's P barrier with the MMA warp
+            if (ok) ok = mbar_wait_warp(&s_full[b], (j >> 1) & 1, abort_flag, p.status);
+            if (!ok) {
+                named_bar_sync(BAR_P, BAR_P_COUNT);
+                continue;
+            }
             tc_fence_after();
             uint32_t s[KT_ROWS];
 #pragma unroll
@@ -309,7 +333,8 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                 if (!mbar_wait_warp(&pv_done[(j - 1) % STAGES], (uint32_t)((j - 1) / STAGES) & 1, abort_flag,
                                     p.status)) {
                     ok = false;
-                    break;
+                    named_bar_sync(BAR_P, BAR_P_COUNT);
+                    continue;
                 }
                 tc_fence_after();
                 {
@@ -334,7 +359,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&p_full[j % STAGES]);
+            named_bar_sync(BAR_P, BAR_P_COUNT);
         }
         if (ok && mbar_wait_warp(&pv_done[(n_tiles - 1) % STAGES], (uint32_t)((n_tiles - 1) / STAGES) & 1, abort_flag,
                                  p.status)) {

@@ -277,6 +277,15 @@ KVB_DEV float fmax3(float a, float b, float c) {
     return d;
 }
 
+// Named barriers (ids 1-15; 0 is __syncthreads): bar.arrive does not block, bar.sync
+// blocks until `count` threads (whole warps) have arrived in the current phase.
+KVB_DEV void named_bar_arrive(uint32_t id, uint32_t count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+KVB_DEV void named_bar_sync(uint32_t id, uint32_t count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 KVB_DEV uint32_t warp_id() { return threadIdx.x >> 5; }
 KVB_DEV uint32_t lane_id() { return threadIdx.x & 31; }
 
