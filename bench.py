@@ -37,7 +37,7 @@ METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % 
 # size (18,713 rows over a 124,032-row cache), from the ncu capture summarised in
 # profiles/attn_kernel_sparse_m18713_nkv124032.md; valid only for the kernel sources it
 # was taken on (sha1 prefixes of attn.cu and common.cuh), otherwise reported as null.
-ATTN_TRAFFIC = {"bytes": 8.170427e9 + 0.141370e9, "sha1": {"attn.cu": "8c11daf63fac", "common.cuh": "90b166ead89b"}}
+ATTN_TRAFFIC = {"bytes": 8.170038e9 + 0.141609e9, "sha1": {"attn.cu": "60fdf53c717a", "common.cuh": "ac1f1dda7832"}}
 
 
 def attn_traffic():
