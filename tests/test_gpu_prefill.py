@@ -198,6 +198,43 @@ def test_full_ratio_equals_dense_prefill(kvb, case):
     case.check_fh(fh.cpu(), case.full_fh, "r = 1 final hidden")
 
 
+def test_zero_ratio_reads_the_realigned_cache(kvb, case):
+    """r = 0: the selective layers recompute only the query rows and every context row
+    keeps its re-aligned chunk cache entry (the plain concatenation baseline of Sec. 4);
+    final hidden and blended caches against the oracle's r = 0 run."""
+    ck, cv = case.new_cache()
+    fh, _, t = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks,
+                                     case.dstarts, case.n_ctx, case.nq, 0.0, 1, ws=case.ws, timings=True)
+    torch.cuda.synchronize()
+    assert kvb.device_status(case.ws) == 0
+    assert t["n_selected"] == 0 and t["n_rows"] == case.nq
+    ref = blend.selective_prefill(case.s, case.l64, case.x0, case.starts, case.nq, 0.0, case.cc["k"], case.cc["v"],
+                                  1, None, case.w["final_norm"])
+    assert len(ref["sel"]) == 0
+    e = case.check_fh(fh.cpu(), ref["final_hidden"], "final hidden (r = 0)")
+    for l in range(case.shape.n_layers):
+        case.check_cache(ck[l].cpu(), ref["k"][l], f"k{l}", f"r = 0 blended K layer {l}")
+        case.check_cache(cv[l].cpu(), ref["v"][l], f"v{l}", f"r = 0 blended V layer {l}")
+    print("r = 0", case.wl.name, e)
+
+
+def test_single_chunk_is_exact_for_any_ratio(kvb):
+    """One chunk at offset 0: its isolated cache is the full prefill's cache (Sec. 1,
+    prefix invariance) and re-alignment is the identity, so the selective prefill gives
+    the full prefill's result whichever rows HKVD picks."""
+    c = Case(kvb, synth.Workload("tiny-2L-1x300+20", synth.TINY, 1, 300, 20))
+    for r in (0.0, 0.15, 0.5):
+        ck, cv = c.new_cache()
+        fh, _, _ = kvb.selective_prefill(c.cfg, c.model, c.rope, c.kch, c.vch, ck, cv, c.dtoks, c.dstarts, c.n_ctx,
+                                         c.nq, r, 1, ws=c.ws)
+        torch.cuda.synchronize()
+        assert kvb.device_status(c.ws) == 0
+        e = c.check_fh(fh.cpu(), c.full_fh, f"single chunk, r = {r}, vs the full prefill")
+        for l in range(c.shape.n_layers):
+            c.check_cache(ck[l].cpu(), c.full["k"][l], f"k{l}", f"single chunk, r = {r}, K layer {l}")
+        print("single chunk r", r, e)
+
+
 def test_repeatable_bitwise(kvb, case):
     """Three runs on the same inputs give bit-identical outputs (no races in the pipeline)."""
     outs = []
