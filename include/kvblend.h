@@ -30,7 +30,8 @@
  *    clear it, kvb_device_status() clears it after reading.
  *
  * Model layout (Llama-3.1 decoder, Sec. 4): hidden H, Hq query heads, Hkv kv heads,
- * head dim D in {64, 128}, MLP dim F, Hq % Hkv == 0 and 128 % (Hq/Hkv) == 0.
+ * head dim D in {64, 128}, MLP dim F, Hq % Hkv == 0 (group sizes Hq/Hkv up to 128 in
+ * the prefill, up to 8 in the decode).
  *  - KV cache of one layer: [n_rows][Hkv][D] for K and for V; a multi-layer cache
  *    is n_layers such blocks back to back.  Row t of the blended cache holds token t
  *    of the concatenated sequence (global position t).  K is bf16.  V holds
