@@ -271,12 +271,20 @@ def test_pipelined_host_ingest_equals_device_resident(kvb, case):
                                    case.dstarts, case.n_ctx, case.nq, case.wl.r, 1)
 
 
-def test_epic_and_kvlink_selection(kvb, case):
+@pytest.fixture(scope="module", params=["tiny_sep", "l8b_1layer_sep"])
+def sep_case(request, kvb):
+    """The workloads with separator tokens between documents (cached with the others)."""
+    if request.param not in _CASES:
+        _CASES[request.param] = Case(kvb, synth.WORKLOADS[request.param])
+    return _CASES[request.param]
+
+
+def test_epic_and_kvlink_selection(kvb, sep_case):
     """Separator workloads: the EPIC set (20 rows from every separator) and the KVLink set
     (the separators) built on the device equal the oracle's; the selective prefill with the
     EPIC set matches the oracle; separator rows left out keep zero K/V in the selective layers."""
-    if not case.sep_rows:
-        pytest.skip("no separators in this workload")
+    case = sep_case
+    assert case.sep_rows
     seps = case.wl.sep_starts()
     dseps = torch.tensor(seps, dtype=torch.int32, device="cuda")
     for window in (20, case.wl.n_sep):
