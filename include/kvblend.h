@@ -253,7 +253,8 @@ kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, const kvb_layer
 
 /* KV scatter (Sec. 3.4: recomputed entries replace the cached ones): for r < m,
  *   k_dst[dst_idx[r]] = k_rows[r], v_dst[dst_idx[r]] = v_rows[r]   (kv_dim elements)
- * dst_idx values must be distinct and < n_dst_rows (bit copy, order irrelevant).
+ * dst_idx values must be distinct and < n_dst_rows (bit copy, order irrelevant); a row
+ * whose dst_idx lies outside [0, n_dst_rows) is skipped (the kernel checks each index).
  * Errors: INVALID_ARG. */
 kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows,
                           const int32_t* dst_idx, int64_t m, int32_t kv_dim,
@@ -304,7 +305,10 @@ kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* byt
  * or NULL (receives the k chosen indices).  t: HOST timings or NULL (timing adds
  * events but no synchronisation until the call returns; with t != NULL the call
  * synchronises the stream once at the end to read the events).  r == 1 computes
- * the dense prefill of every layer.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
+ * the dense prefill of every layer.  Device-side checks: a token id outside [0, vocab)
+ * embeds as a zero row and a forced_sel entry outside [0, n_ctx) is replaced by row 0;
+ * both record KVB_ERR_INVALID_ARG in the workspace status word (kvb_device_status), and
+ * the results of such a call are not meaningful.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
 kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
                                  const kvb_rope_table* rope,
                                  const uint16_t* k_chunks, const uint16_t* v_chunks,
@@ -352,7 +356,9 @@ kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, i
  *   (NULL = t).  With kv_lo = chunk start and rope_pos = t - chunk start every chunk
  *   is prefilled alone at chunk-local positions.
  * Writes every layer's K/V into cache rows [0, n) and, if final_hidden != NULL, the
- * final RMSNorm of the last n_out rows to final_hidden [n_out][H].  Errors as above. */
+ * final RMSNorm of the last n_out rows to final_hidden [n_out][H].  Token ids outside
+ * [0, vocab) are reported in the status word as for kvb_selective_prefill.  Errors as
+ * above. */
 kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
                             const kvb_rope_table* rope, kvb_kv_cache* cache,
                             const int32_t* token_ids, int64_t n,

@@ -535,7 +535,8 @@ kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const 
     KVB_TRY(check_ptr(dst_idx, "dst_idx"));
     KVB_TRY(check_ptr(k_dst, "k_dst"));
     KVB_TRY(check_ptr(v_dst, "v_dst"));
-    return launch_scatter(k_rows, v_rows, dst_idx, m, kv_dim, k_dst, v_dst, static_cast<cudaStream_t>(stream));
+    return launch_scatter(k_rows, v_rows, dst_idx, m, kv_dim, k_dst, v_dst, n_dst_rows,
+                          static_cast<cudaStream_t>(stream));
 }
 
 kvb_status kvb_sparse_query_attn(const kvb_config* cfg, const uint16_t* q, const int32_t* q_idx,
@@ -613,7 +614,7 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
     tm.start(t != nullptr, c.st);
     const int64_t kvd = c.KVD;
     KVB_TRY(launch_iota(w.ident, n, 0, c.st));
-    KVB_TRY(launch_embed(model->embed, token_ids, n, c.H, w.x_all, c.st));
+    KVB_TRY(launch_embed(model->embed, token_ids, n, c.H, cfg->vocab, w.x_all, w.status, c.st));
     for (int l = 0; l < cfg->n_layers; ++l) {
         uint16_t* kc = cache->k + (int64_t)l * cache->n_rows * kvd;
         uint16_t* vc = cache->v + (int64_t)l * cache->n_rows * kvd;
@@ -753,7 +754,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
     tm.mark();
     // 2. dense layers (layer 0 at least): every row, causal
     KVB_TRY(launch_iota(w.ident, N, 0, c.st));
-    KVB_TRY(launch_embed(model->embed, token_ids, N, c.H, w.x_all, c.st));
+    KVB_TRY(launch_embed(model->embed, token_ids, N, c.H, cfg->vocab, w.x_all, w.status, c.st));
     for (int l = 0; l < lc; ++l)
         KVB_TRY(layer(c, &model->layers[l], w.x_all, N, nullptr, w.ident, nullptr, kc(l), vc(l), N));
     tm.mark();
@@ -780,7 +781,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
             sel = w.sel;
         }
         m = k + n_query;
-        KVB_TRY(launch_concat_rows(sel, k, n_ctx, n_query, w.rows, c.st));
+        KVB_TRY(launch_concat_rows(sel, k, n_ctx, n_query, w.rows, w.status, c.st));
         KVB_TRY(launch_gather_rows(w.x_all, w.rows, m, c.H, w.x_sel, c.st));
         if (sel_out && k > 0)
             KVB_TRY(cuda_ok(cudaMemcpyAsync(sel_out, sel, (size_t)k * 4, cudaMemcpyDeviceToDevice, c.st), "sel copy"));

@@ -82,16 +82,22 @@ realign_kernel(const float* __restrict__ cos_t, const float* __restrict__ sin_t,
 
 // ------------------------------------------------------------------ embedding
 __global__ void __launch_bounds__(256)
-embed_kernel(const uint16_t* __restrict__ embed, const int32_t* __restrict__ tok, int64_t n, int H,
-             float* __restrict__ x) {
+embed_kernel(const uint16_t* __restrict__ embed, const int32_t* __restrict__ tok, int64_t n, int H, int vocab,
+             float* __restrict__ x, int* status) {
     const int vec = H / 8;
     const int64_t items = n * vec;
     for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < items;
          it += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = it / vec;
         const int c = (int)(it - r * vec);
-        const uint4 e = __ldg(reinterpret_cast<const uint4*>(embed + (int64_t)__ldg(tok + r) * H) + c);
+        const int32_t t = __ldg(tok + r);
         float4* dst = reinterpret_cast<float4*>(x + r * H) + 2 * c;
+        if ((uint32_t)t >= (uint32_t)vocab) {   // outside the table: a zero row, reported
+            if (c == 0) set_status(status, KVB_ERR_INVALID_ARG);
+            dst[0] = dst[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+            continue;
+        }
+        const uint4 e = __ldg(reinterpret_cast<const uint4*>(embed + (int64_t)t * H) + c);
         dst[0] = make_float4(bf16_lo(e.x), bf16_hi(e.x), bf16_lo(e.y), bf16_hi(e.y));
         dst[1] = make_float4(bf16_lo(e.z), bf16_hi(e.z), bf16_lo(e.w), bf16_hi(e.w));
     }
@@ -158,7 +164,7 @@ gather_rows_kernel(const float* __restrict__ src, const int32_t* __restrict__ id
 __global__ void __launch_bounds__(256)
 scatter_kernel(const uint16_t* __restrict__ k_rows, const uint16_t* __restrict__ v_rows,
                const int32_t* __restrict__ dst_idx, int64_t m, int kv_dim, uint16_t* __restrict__ k_dst,
-               uint16_t* __restrict__ v_dst) {
+               uint16_t* __restrict__ v_dst, int64_t n_dst) {
     const int vec = kv_dim / 8;
     const int64_t items = m * vec;
     for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < items;
@@ -166,6 +172,7 @@ scatter_kernel(const uint16_t* __restrict__ k_rows, const uint16_t* __restrict__
         const int64_t r = it / vec;
         const int c = (int)(it - r * vec);
         const int64_t d = __ldg(dst_idx + r);
+        if (d < 0 || d >= n_dst) continue;   // outside the destination: skipped
         reinterpret_cast<uint4*>(k_dst + d * kv_dim)[c] = reinterpret_cast<const uint4*>(k_rows + r * kv_dim)[c];
         reinterpret_cast<uint4*>(v_dst + d * kv_dim)[c] = reinterpret_cast<const uint4*>(v_rows + r * kv_dim)[c];
     }
@@ -176,11 +183,22 @@ __global__ void iota_kernel(int32_t* out, int64_t n, int32_t start) {
         out[i] = start + (int32_t)i;
 }
 
-// rows = [sel[0..k) , n_ctx .. n_ctx + n_query)
-__global__ void concat_rows_kernel(const int32_t* sel, int64_t k, int64_t n_ctx, int64_t n_query, int32_t* rows) {
+// rows = [sel[0..k) , n_ctx .. n_ctx + n_query); a selected index outside [0, n_ctx) is
+// reported and replaced by row 0, so that no later gather or scatter leaves the buffers
+__global__ void concat_rows_kernel(const int32_t* sel, int64_t k, int64_t n_ctx, int64_t n_query, int32_t* rows,
+                                   int* status) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < k + n_query;
-         i += (int64_t)gridDim.x * blockDim.x)
-        rows[i] = i < k ? sel[i] : (int32_t)(n_ctx + (i - k));
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int32_t v = (int32_t)(n_ctx + (i - k));
+        if (i < k) {
+            v = sel[i];
+            if (v < 0 || v >= n_ctx) {
+                set_status(status, KVB_ERR_INVALID_ARG);
+                v = 0;
+            }
+        }
+        rows[i] = v;
+    }
 }
 
 unsigned grid_for(int64_t items, int threads) {
@@ -210,9 +228,11 @@ kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv
     return cuda_ok(cudaGetLastError(), "realign launch");
 }
 
-kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, float* x, cudaStream_t st) {
+kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, int vocab, float* x,
+                        int* status, cudaStream_t st) {
     if (n <= 0) return KVB_OK;
-    embed_kernel<<<grid_for(n * (H / 8), 256), 256, 0, st>>>(embed, tok, n, H, x);
+    if (vocab < 1) return fail(KVB_ERR_INVALID_ARG, "embedding: vocab %d < 1", vocab);
+    embed_kernel<<<grid_for(n * (H / 8), 256), 256, 0, st>>>(embed, tok, n, H, vocab, x, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "embed launch");
 }
@@ -242,9 +262,10 @@ kvb_status launch_gather_rows(const float* src, const int32_t* idx, int64_t m, i
 }
 
 kvb_status launch_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const int32_t* dst_idx, int64_t m,
-                          int kv_dim, uint16_t* k_dst, uint16_t* v_dst, cudaStream_t st) {
+                          int kv_dim, uint16_t* k_dst, uint16_t* v_dst, int64_t n_dst, cudaStream_t st) {
     if (m <= 0) return KVB_OK;
-    scatter_kernel<<<grid_for(m * (kv_dim / 8), 256), 256, 0, st>>>(k_rows, v_rows, dst_idx, m, kv_dim, k_dst, v_dst);
+    scatter_kernel<<<grid_for(m * (kv_dim / 8), 256), 256, 0, st>>>(k_rows, v_rows, dst_idx, m, kv_dim, k_dst, v_dst,
+                                                                   n_dst);
     count_launch();
     return cuda_ok(cudaGetLastError(), "scatter launch");
 }
@@ -257,9 +278,9 @@ kvb_status launch_iota(int32_t* out, int64_t n, int32_t start, cudaStream_t st) 
 }
 
 kvb_status launch_concat_rows(const int32_t* sel, int64_t k, int64_t n_ctx, int64_t n_query, int32_t* rows,
-                              cudaStream_t st) {
+                              int* status, cudaStream_t st) {
     if (k + n_query <= 0) return KVB_OK;
-    concat_rows_kernel<<<grid_for(k + n_query, 256), 256, 0, st>>>(sel, k, n_ctx, n_query, rows);
+    concat_rows_kernel<<<grid_for(k + n_query, 256), 256, 0, st>>>(sel, k, n_ctx, n_query, rows, status);
     count_launch();
     return cuda_ok(cudaGetLastError(), "rows launch");
 }

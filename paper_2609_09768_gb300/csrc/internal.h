@@ -85,16 +85,20 @@ kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv
                           const uint16_t* v_src, int64_t src_layer_stride, uint16_t* k_dst, uint16_t* v_dst,
                           int64_t dst_layer_stride, int n_layers, const int32_t* chunk_start, int n_chunks,
                           int64_t n_ctx, cudaStream_t st);
-kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, float* x, cudaStream_t st);
+// token ids outside [0, vocab) give a zero row and KVB_ERR_INVALID_ARG in *status
+kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, int vocab, float* x,
+                        int* status, cudaStream_t st);
 // out_bf16[r] / out_f32[r] = RMSNorm(x[idx ? idx[r] : r]) * g   (one of the outputs may be NULL)
 kvb_status launch_rmsnorm(const float* x, const int32_t* idx, int64_t m, int H, const float* g, float eps,
                           uint16_t* out_bf16, float* out_f32, cudaStream_t st);
 kvb_status launch_gather_rows(const float* src, const int32_t* idx, int64_t m, int H, float* dst, cudaStream_t st);
+// rows with dst_idx outside [0, n_dst) are skipped
 kvb_status launch_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const int32_t* dst_idx, int64_t m,
-                          int kv_dim, uint16_t* k_dst, uint16_t* v_dst, cudaStream_t st);
+                          int kv_dim, uint16_t* k_dst, uint16_t* v_dst, int64_t n_dst, cudaStream_t st);
 kvb_status launch_iota(int32_t* out, int64_t n, int32_t start, cudaStream_t st);
+// sel entries outside [0, n_ctx) become row 0 and KVB_ERR_INVALID_ARG in *status
 kvb_status launch_concat_rows(const int32_t* sel, int64_t k, int64_t n_ctx, int64_t n_query, int32_t* rows,
-                              cudaStream_t st);
+                              int* status, cudaStream_t st);
 
 // ---------------------------------------------------------------- HKVD + top-k
 size_t hkvd_ws_bytes(int64_t n_ctx);

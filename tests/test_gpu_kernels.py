@@ -221,6 +221,76 @@ def test_kv_scatter_bit_exact(kvb, m, kv_dim, n_dst):
     assert torch.equal(kd.cpu(), want_k) and torch.equal(vd.cpu(), want_v)
 
 
+def test_kv_scatter_skips_rows_outside_the_destination(kvb):
+    """A destination index outside [0, n_dst_rows) is skipped, not written.  The
+    destination is a view of the first rows of a larger buffer, so the row just past
+    it is memory of this test and must stay untouched."""
+    n_dst, kv_dim = 6, 128
+    kr = synth.randn_bf16((3, kv_dim), 411)
+    vr = synth.randn_bf16((3, kv_dim), 412).to(torch.float16)
+    idx = torch.tensor([1, n_dst, 4], dtype=torch.int32)
+    kpad = torch.zeros(n_dst + 1, kv_dim, dtype=torch.bfloat16, device="cuda")
+    vpad = torch.zeros(n_dst + 1, kv_dim, dtype=torch.float16, device="cuda")
+    kvb.kv_scatter(dev(kr), dev(vr), dev(idx), kpad[:n_dst], vpad[:n_dst])
+    torch.cuda.synchronize()
+    want_k = torch.zeros(n_dst + 1, kv_dim, dtype=torch.bfloat16)
+    want_v = torch.zeros(n_dst + 1, kv_dim, dtype=torch.float16)
+    want_k[[1, 4]] = kr[[0, 2]]
+    want_v[[1, 4]] = vr[[0, 2]]
+    assert torch.equal(kpad.cpu(), want_k) and torch.equal(vpad.cpu(), want_v)
+
+
+def _tiny_device_model(kvb, pad_embed_rows=0):
+    w = synth.make_model(TINY, 0)
+    emb = torch.zeros(TINY.vocab + pad_embed_rows, TINY.hidden, dtype=torch.bfloat16, device="cuda")
+    emb[: TINY.vocab] = w["embed"].cuda()
+    return kvb.Model({"layers": [{k: v.cuda() for k, v in l.items()} for l in w["layers"]],
+                      "embed": emb[: TINY.vocab], "final_norm": w["final_norm"].cuda()})
+
+
+def test_token_ids_outside_the_vocabulary_are_reported(kvb):
+    """A token id outside [0, vocab) embeds as a zero row and sets KVB_ERR_INVALID_ARG in
+    the status word; the next valid call reports nothing.  The embedding table is a view
+    of a larger buffer, so the row just past the vocabulary is memory of this test."""
+    cfg = kvb.config(TINY)
+    model = _tiny_device_model(kvb, pad_embed_rows=1)
+    n = 40
+    rope = kvb.RopeTable(cfg, n)
+    toks = synth.make_tokens(TINY, n, 3).cuda()
+    ck = torch.zeros(TINY.n_layers, n, TINY.n_kv_heads, TINY.head_dim, dtype=torch.bfloat16, device="cuda")
+    cv = torch.zeros(ck.shape, dtype=torch.float16, device="cuda")
+    ws = kvb.workspace(cfg, n)
+    bad = toks.clone()
+    bad[7] = TINY.vocab
+    kvb.full_prefill(cfg, model, rope, ck, cv, bad, n_out=1, ws=ws)
+    assert kvb.device_status(ws) == kvb.KVB_ERR_INVALID_ARG
+    fh, _ = kvb.full_prefill(cfg, model, rope, ck, cv, toks, n_out=1, ws=ws)
+    assert kvb.device_status(ws) == kvb.KVB_OK
+    assert torch.isfinite(fh).all()
+
+
+def test_forced_selection_outside_the_context_is_reported(kvb):
+    """A forced selected row outside [0, n_ctx) is reported as KVB_ERR_INVALID_ARG in the
+    status word and replaced by row 0 (row n_ctx, the one named here, exists in the
+    workspace and the cache, so nothing outside them is touched either way)."""
+    wl = synth.WORKLOADS["tiny"]
+    cfg = kvb.config(TINY)
+    model = _tiny_device_model(kvb)
+    rope = kvb.RopeTable(cfg, wl.n_total)
+    toks = wl.tokens().cuda()
+    kch = torch.zeros(TINY.n_layers, wl.n_ctx, TINY.n_kv_heads, TINY.head_dim, dtype=torch.bfloat16, device="cuda")
+    vch = torch.zeros(kch.shape, dtype=torch.float16, device="cuda")
+    ck = torch.zeros(TINY.n_layers, wl.n_total, TINY.n_kv_heads, TINY.head_dim, dtype=torch.bfloat16, device="cuda")
+    cv = torch.zeros(ck.shape, dtype=torch.float16, device="cuda")
+    starts = torch.tensor(wl.chunk_starts(), dtype=torch.int32, device="cuda")
+    ws = kvb.workspace(cfg, wl.n_total)
+    for forced, want in (([3, 9, wl.n_ctx], kvb.KVB_ERR_INVALID_ARG), ([3, 9, wl.n_ctx - 1], kvb.KVB_OK)):
+        sel = torch.tensor(forced, dtype=torch.int32, device="cuda")
+        kvb.selective_prefill(cfg, model, rope, kch, vch, ck, cv, toks, starts, wl.n_ctx, wl.n_query, 0.0, 1,
+                              forced_sel=sel, ws=ws)
+        assert kvb.device_status(ws) == want
+
+
 def test_bounded_wait_reports_timeout_and_context_survives(kvb):
     """A wait that nothing completes gives up after its limit and reports KVB_ERR_TIMEOUT
     through the status word; the context stays usable and the word is cleared on read."""
