@@ -31,12 +31,11 @@ token index; the residual stream is kept in full precision.
 from __future__ import annotations
 
 import math
-from typing import Optional, Sequence
+from typing import Sequence
 
 import numpy as np
 
-from .llama import (F64, Shape, act, as64, apply_rope, attn_out_mlp, k_rows, layer_rows,
-                    rmsnorm, rope_cos_sin)
+from .llama import (F64, Shape, act, as64, apply_rope, k_rows, layer_rows, rmsnorm, rope_cos_sin)
 
 
 def embed_rows(embed, tokens) -> np.ndarray:

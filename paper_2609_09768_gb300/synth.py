@@ -24,7 +24,7 @@ one layer can be regenerated without drawing the others.
 from __future__ import annotations
 
 import dataclasses
-from typing import Dict, List, Optional, Sequence
+from typing import Dict, List, Sequence
 
 import torch
 
