@@ -34,9 +34,9 @@ sys.path.insert(0, ROOT)
 METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % of bf16 peak"
 
 # DRAM bytes (read + write) per launch of the selective-layer attention at this workload's
-# size (18,713 rows over a 124,032-row cache), from the ncu capture summarised in
-# profiles/attn_kernel_sparse_m18713_nkv124032.md; valid only for the kernel sources it
-# was taken on (sha1 prefixes of attn.cu and common.cuh), otherwise reported as null.
+# size (18,713 rows over a 124,032-row cache), from one ncu capture of that launch; valid
+# only for the kernel sources it was taken on (sha1 prefixes of attn.cu and common.cuh),
+# otherwise reported as null.
 ATTN_TRAFFIC = {"bytes": 8.170038e9 + 0.141609e9, "sha1": {"attn.cu": "60fdf53c717a", "common.cuh": "ac1f1dda7832"}}
 
 
@@ -68,6 +68,17 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--sweep", action="store_true",
                     help="64k-context sweep: r x chunk size, per-kernel times (prints one JSON line per point)")
+    ap.add_argument("--kernel", default=None,
+                    choices=["attn", "dense", "gemm", "realign", "decode_attn", "decode_step"],
+                    help="time one kernel of the library on a seeded synthetic Llama-3.1-8B-shaped case "
+                         "(for ncu captures); prints one JSON line")
+    ap.add_argument("--m", type=int, default=18713, help="--kernel attn / gemm: query rows")
+    ap.add_argument("--n-kv", type=int, default=124032, help="--kernel attn / dense / decode_*: cache rows")
+    ap.add_argument("--n-ctx", type=int, default=123904, help="--kernel realign: context rows")
+    ap.add_argument("--layers", type=int, default=2, help="--kernel realign / decode_step: layers")
+    ap.add_argument("--which", default="qkv", choices=["qkv", "o", "gateup", "down"], help="--kernel gemm")
+    ap.add_argument("--reps", type=int, default=2, help="--kernel: calls, the last one timed")
+    ap.add_argument("--timed", type=int, default=1, help="--kernel: calls between the timing events (mean)")
     ap.add_argument("--selectors", action="store_true",
                     help="separator workload: TTFT and per-layer key-deviation histograms against the full "
                          "prefill for plain concatenation, HKVD, EPIC and KVLink selections (one JSON line each)")
@@ -380,7 +391,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         e2e_ms = a.elapsed_time(b) / args.e2e_steps
         # the bare host->device copy of the same caches, for reference
         kd = torch.empty_like(kch)
-        a.record(); kd.copy_(hk, non_blocking=True); kd.copy_(hv.view(torch.bfloat16), non_blocking=True); b.record()
+        a.record(); kd.copy_(hk, non_blocking=True); kd.copy_(hv, non_blocking=True); b.record()
         torch.cuda.synchronize()
         h2d_ms = a.elapsed_time(b)
         h2d = hk.numel() * 2 + hv.numel() * 2 + ht.numel() * 4
@@ -602,8 +613,123 @@ def run_selectors(args) -> None:
     assert kvb.device_status(ws) == 0
 
 
+def run_kernel(args) -> None:
+    """One kernel on a seeded synthetic case of the Llama-3.1-8B layer shape (H 4096, 32 q / 8
+    kv heads, D 128, F 14336).  attn: --m query rows drawn uniformly over the cache (as the
+    HKVD choice at r = m / n_kv would spread them) plus the last row; dense: causal over all
+    --n-kv rows; gemm: the QKV GEMM or the back half of a layer on --m rows; realign: --layers
+    layers of --n-ctx rows of chunk caches in 512-row chunks; decode_attn / decode_step: one
+    decode row at position --n-kv - 1.  Prints the CUDA-event time of the last call (or the
+    mean of --timed calls) and its algorithmic throughput."""
+    import torch
+    from paper_2609_09768_gb300 import build, synth
+    from paper_2609_09768_gb300 import kvblend as kvb
+    build.build()
+    shape = synth.LLAMA8B
+    cfg = kvb.config(shape)
+    dev = torch.device("cuda")
+    Hq, Hkv, D, H, F = shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.hidden, shape.mlp_dim
+    g = torch.Generator(device=dev)
+    g.manual_seed(0)
+    ws = torch.zeros(256, dtype=torch.uint8, device=dev)
+    out, flop = {}, None
+    if args.kernel in ("attn", "dense"):
+        n_kv = args.n_kv
+        if args.kernel == "dense":
+            rows = torch.arange(n_kv, device=dev, dtype=torch.int32)
+        else:
+            perm = torch.randperm(n_kv - 1, generator=g, device=dev)[: args.m - 1]
+            rows = torch.cat([torch.sort(perm).values, torch.tensor([n_kv - 1], device=dev)]).to(torch.int32)
+        m = rows.numel()
+        q = torch.randn(m, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        kc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16).to(torch.float16)
+        o = torch.empty(m, Hq * D, dtype=torch.bfloat16, device=dev)
+        fn = lambda: kvb.sparse_query_attn(cfg, q, rows, None, kc, vc, o, ws)
+        flop = 4.0 * Hq * D * float((rows.to(torch.float64) + 1).sum())
+        out.update(m=m, n_kv=n_kv)
+    elif args.kernel == "gemm":
+        m = args.m
+        lws = kvb.layer_struct(synth.make_layer_weights(shape, 0, 0, dev))
+        wsl = kvb.workspace(cfg, m, dev)
+        if args.which == "qkv":
+            x = torch.randn(m, H, generator=g, device=dev)
+            pos = torch.arange(m, dtype=torch.int32, device=dev)
+            rope = kvb.RopeTable(cfg, m, dev)
+            qo = torch.empty(m, Hq * D, dtype=torch.bfloat16, device=dev)
+            ko = torch.empty(m, Hkv * D, dtype=torch.bfloat16, device=dev)
+            vo = torch.empty(m, Hkv * D, dtype=torch.float16, device=dev)
+            fn = lambda: kvb.gather_rmsnorm_qkv(cfg, lws, rope, x, None, pos, m, qo, ko, vo, None, wsl)
+            flop = 2.0 * m * H * shape.qkv_dim
+        else:
+            attn = torch.randn(m, Hq * D, generator=g, device=dev).to(torch.bfloat16)
+            x = torch.randn(m, H, generator=g, device=dev)
+            fn = lambda: kvb.mlp_rows(cfg, lws, attn, x, wsl)
+            flop = 2.0 * m * H * (Hq * D + 3 * F)
+        out.update(m=m, which=("o+gateup+down (mlp_rows)" if args.which != "qkv" else "qkv"))
+    elif args.kernel == "decode_attn":
+        n_kv = args.n_kv
+        q = torch.randn(Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        kc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn(n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16).to(torch.float16)
+        pos = torch.tensor([n_kv - 1], dtype=torch.int32, device=dev)
+        ws = kvb.decode_workspace(cfg, n_kv, dev)
+        o = torch.empty(Hq, D, dtype=torch.bfloat16, device=dev)
+        fn = lambda: kvb.decode_attention(cfg, q, kc, vc, pos, n_kv, out=o, ws=ws)
+        out.update(bytes=float(n_kv) * Hkv * D * 2 * 2, n_kv=n_kv)
+    elif args.kernel == "decode_step":
+        # a decode step of a --layers-layer model at position n_kv - 1
+        shp = shape.with_layers(args.layers)
+        cfgl = kvb.config(shp)
+        model = kvb.Model(synth.make_model(shp, 0, dev))
+        lm = synth.make_lm_head(shp, 0, dev)
+        n_kv = args.n_kv
+        rope = kvb.RopeTable(cfgl, n_kv, dev)
+        kc = torch.randn(args.layers, n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vc = torch.randn(args.layers, n_kv, Hkv, D, generator=g, device=dev).to(torch.bfloat16).to(torch.float16)
+        tokens = torch.zeros(n_kv + 1, dtype=torch.int32, device=dev)
+        pos = torch.tensor([n_kv - 1], dtype=torch.int32, device=dev)
+        ws = kvb.decode_workspace(cfgl, n_kv, dev)
+
+        def fn():
+            pos.fill_(n_kv - 1)
+            kvb.decode_step(cfgl, model, rope, kc, vc, lm, tokens, pos, n_kv, ws=ws)
+        wb = args.layers * 2.0 * (shp.qkv_dim * H + H * shp.q_dim + 3 * H * F) + shp.vocab * H * 2.0
+        out.update(bytes=wb + args.layers * float(n_kv) * Hkv * D * 4, layers=args.layers, n_kv=n_kv)
+    else:
+        L, n_ctx = args.layers, args.n_ctx
+        ks = torch.randn(L, n_ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vs = torch.randn(L, n_ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        kd = torch.empty_like(ks)
+        vd = torch.empty(vs.shape, dtype=torch.float16, device=dev)
+        rope = kvb.RopeTable(cfg, n_ctx, dev)
+        starts = torch.arange(0, n_ctx + 1, 512, dtype=torch.int32, device=dev)
+        fn = lambda: kvb.rope_realign(cfg, rope, ks, vs, kd, vd, 0, L, starts, n_ctx, ws=ws)
+        out.update(bytes=4.0 * ks.numel() * 2, layers=L, n_ctx=n_ctx)
+    for _ in range(args.reps - 1):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(max(args.timed, 1)):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / max(args.timed, 1)
+    assert kvb.device_status(ws) == 0
+    out.update(kernel=args.kernel, ms=round(ms, 4))
+    if flop:
+        out["tflops"] = round(flop / (ms * 1e-3) / 1e12, 1)
+    if "bytes" in out:
+        out["gbs"] = round(out["bytes"] / (ms * 1e-3) / 1e9, 1)
+    print(json.dumps(out))
+
+
 def main():
     args = parse()
+    if args.kernel:
+        run_kernel(args)
+        return
     from paper_2609_09768_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
     if args.model_config:

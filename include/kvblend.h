@@ -33,12 +33,21 @@
  * head dim D in {64, 128}, MLP dim F, Hq % Hkv == 0 (group sizes Hq/Hkv up to 128 in
  * the prefill, up to 8 in the decode).
  *  - KV cache of one layer: [n_rows][Hkv][D] for K and for V; a multi-layer cache
- *    is n_layers such blocks back to back.  Row t of the blended cache holds token t
- *    of the concatenated sequence (global position t).  K is bf16.  V holds
- *    bf16-precision values (the paper's bf16 KV cache) in fp16 containers, so that
- *    the attention's P.V product runs as an fp16 MMA whose softmax weights are
- *    rounded to fp16 rather than bf16 (8x smaller rounding error, same speed).
- *    Converting a bf16 V cache to this layout is exact.
+ *    is n_layers such blocks back to back.  Two formats:
+ *      chunk caches (what a caller stores per document, Sec. 3.4: the inputs of
+ *      kvb_rope_realign and kvb_selective_prefill*, the optional V output of
+ *      kvb_full_prefill): K and V both bf16, as the paper's bf16 model writes them;
+ *      the blended cache (row t holds token t of the concatenated sequence, global
+ *      position t; what the attention kernels read): K bf16, V in fp16 containers
+ *      holding bf16-precision values, so that the attention's P.V product runs as an
+ *      fp16 MMA whose softmax weights are rounded to fp16 rather than bf16 (8x
+ *      smaller rounding error, same speed).
+ *    The bf16 -> fp16 conversion of V (done by the merge pass, which reads and writes
+ *    every V element anyway) is exact for 2^-14 <= |v| <= 65504 and for 0; a smaller
+ *    non-zero |v| is rounded to fp16's subnormal spacing 2^-24 (absolute error at most
+ *    2^-25); |v| > 65504 (the largest bf16 value below it is 65280) cannot be held:
+ *    it is written as +-65504, NaN stays NaN, and both record KVB_ERR_RANGE in the
+ *    workspace status word.
  *  - RoPE is rotate-half (dimension i pairs with i + D/2); tables hold
  *    cos/sin(pos * w_i) in fp32, [max_pos][D/2], computed in double precision.
  */
@@ -58,7 +67,9 @@ typedef enum kvb_status {
     KVB_ERR_UNSUPPORTED = 2,   /* valid in principle but not built (e.g. head_dim 96)   */
     KVB_ERR_CUDA = 3,          /* a CUDA runtime/driver call or a launch failed         */
     KVB_ERR_TIMEOUT = 4,       /* device side: a bounded wait in a kernel ran out       */
-    KVB_ERR_WORKSPACE = 5      /* workspace missing or smaller than required            */
+    KVB_ERR_WORKSPACE = 5,     /* workspace missing or smaller than required            */
+    KVB_ERR_RANGE = 6          /* device side: a value outside the range of its storage
+                                * type (a V entry beyond fp16's finite range)           */
 } kvb_status;
 
 /* Frequency scaling of the rotary embedding (kvb_config.rope_scaling). */
@@ -114,8 +125,8 @@ typedef struct kvb_rope_table {
     int64_t max_pos;
 } kvb_rope_table;
 
-/* Multi-layer KV cache: k (bf16) and v (fp16, bf16-precision values) are
- * [n_layers][n_rows][Hkv][D]. */
+/* Multi-layer blended KV cache: k (bf16) and v (fp16 containers, bf16-precision values)
+ * are [n_layers][n_rows][Hkv][D]. */
 typedef struct kvb_kv_cache {
     uint16_t* k;
     uint16_t* v;
@@ -141,6 +152,28 @@ typedef struct kvb_timings {
     int64_t n_selected;   /* k = number of recomputed context rows                   */
     int64_t n_rows;       /* m = k + n_query                                          */
 } kvb_timings;
+
+/* Residual rows captured at layer boundaries, for inspection and per-layer parity checks
+ * (the paper has no counterpart).  For every i < n, the fp32 residual rows that ENTER
+ * layer layers[i] are copied into x_out + i * rows_cap * H just before that layer runs;
+ * layers[i] == n_layers captures the rows leaving the last layer (before the final
+ * RMSNorm).  Which rows: in a dense layer (every layer of kvb_full_prefill; the layers
+ * before check_layer of a selective prefill, or all of them when it runs dense) all rows
+ * in sequence order; from check_layer on, the m = k + n_query recomputed rows: the
+ * selected context rows in ascending index order (as sel_out), then the query rows.
+ * The copies run on the call's stream (device to device), outside any kernel.
+ *   layers:   HOST int32 [n], each in [0, n_layers], any order, repeats allowed
+ *   x_out:    DEVICE fp32 [n][rows_cap][H], 16-byte aligned
+ *   rows_cap: rows per slot; a tap that needs more rows fails the call with INVALID_ARG
+ *             before anything is launched
+ *   rows_out: HOST int64 [n] or NULL: the number of rows captured for layers[i] */
+typedef struct kvb_layer_taps {
+    int32_t n;
+    const int32_t* layers;
+    float* x_out;
+    int64_t rows_cap;
+    int64_t* rows_out;
+} kvb_layer_taps;
 
 /* ------------------------------------------------------------------ status */
 
@@ -175,19 +208,25 @@ kvb_status kvb_attention_scale(const kvb_config* cfg, float* scale_out);
  * adjustment"; PIE, Sec. 2).  For layers [layer_begin, layer_end) and every context
  * row t < n_ctx in chunk c (chunk_start[c] <= t < chunk_start[c+1]):
  *   k_dst[l][t] = R(chunk_start[c]) k_src[l][t]   (rotation of every head's pairs by
- *                                                  the chunk offset, fp32 math)
- *   v_dst[l][t] = v_src[l][t]                     (skipped when v_src == v_dst or NULL)
- * k_src/v_src are [n_layers][src_rows][Hkv][D] (K bf16, V fp16) with keys rotated at chunk-local
- * positions; k_dst/v_dst are [n_layers][dst_rows][Hkv][D].  In place is allowed
- * (k_src == k_dst, src_rows == dst_rows).  chunk_start: DEVICE int32 [n_chunks+1],
- * ascending, chunk_start[0] == 0, chunk_start[n_chunks] == n_ctx.  The rope table
- * must cover max_pos > chunk_start[n_chunks-1].  Errors: INVALID_ARG. */
+ *                                                  the chunk offset, fp32 math, bf16 out)
+ *   v_dst[l][t] = v_src[l][t]                     (bf16 chunk format -> fp16 container of
+ *                                                  the blended cache; skipped when v_src or
+ *                                                  v_dst is NULL)
+ * k_src/v_src are chunk caches [n_layers][src_rows][Hkv][D] (K and V bf16) with keys
+ * rotated at chunk-local positions; k_dst/v_dst are blended-cache layers
+ * [n_layers][dst_rows][Hkv][D] (K bf16, V fp16).  In place is allowed (k_src == k_dst,
+ * v_src == v_dst, src_rows == dst_rows: V is then converted in place).  chunk_start:
+ * DEVICE int32 [n_chunks+1], ascending, chunk_start[0] == 0, chunk_start[n_chunks] ==
+ * n_ctx.  The rope table must cover max_pos > chunk_start[n_chunks-1].  ws: at least 256
+ * bytes whose first word is the device status word, which receives KVB_ERR_RANGE if a V
+ * value lies outside fp16's range (see the layout notes above); may be NULL when V is
+ * skipped.  Errors: INVALID_ARG, WORKSPACE. */
 kvb_status kvb_rope_realign(const kvb_config* cfg, const kvb_rope_table* rope,
                             const uint16_t* k_src, const uint16_t* v_src, int64_t src_rows,
                             uint16_t* k_dst, uint16_t* v_dst, int64_t dst_rows,
                             int32_t layer_begin, int32_t layer_end,
                             const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
-                            void* stream);
+                            void* ws, size_t ws_bytes, void* stream);
 
 /* Workspace bytes kvb_hkvd_select needs for n_ctx rows. */
 size_t kvb_hkvd_workspace_size(int64_t n_ctx);
@@ -212,19 +251,23 @@ kvb_status kvb_hkvd_select(const uint16_t* k_fresh, int64_t ld_fresh,
  * decoder layer, Sec. 4 model):
  *   a[r]   = RMSNorm(x[row_idx[r]]) * attn_norm          (x: fp32 [*][H]; row_idx NULL = r)
  *   q[r]   = RoPE(a[r] W_q^T, rope_pos[r])  -> q_out [m][Hq D] bf16
- *   k[r]   = RoPE(a[r] W_k^T, rope_pos[r])  -> k_out row kv_dst[r] (or r), [*][Hkv D] bf16
+ *   k[r]   = RoPE(a[r] W_k^T, rope_pos[r])  -> k_out row kv_dst[r] (or r), [n_kv_rows][Hkv D] bf16
  *   v[r]   = a[r] W_v^T                     -> v_out row kv_dst[r] (or r), fp16 holding
  *                                              the bf16-rounded value
  * Passing a cache layer as k_out/v_out with kv_dst = the rows' cache indices fuses the
- * KV scatter.  rope_pos: [m] int32 (< rope->max_pos).  Uses tcgen05 tensor cores
- * (bf16 in, fp32 accumulate).  Workspace >= kvb_workspace_size(cfg, m).  Errors:
- * INVALID_ARG, WORKSPACE, UNSUPPORTED. */
+ * KV scatter.  rope_pos: [m] int32.  Index contents are checked on the device where they
+ * are used: a row whose destination kv_dst[r] (or r) lies outside [0, n_kv_rows) writes
+ * no k/v row, and a rope_pos[r] outside [0, rope->max_pos) is rotated by position 0;
+ * either records KVB_ERR_INVALID_ARG in the workspace status word (the results of such
+ * a call are not meaningful, but no memory outside the given buffers is touched).  Uses
+ * tcgen05 tensor cores (bf16 in, fp32 accumulate).  Workspace >= kvb_workspace_size(cfg,
+ * m).  Errors: INVALID_ARG, WORKSPACE, UNSUPPORTED. */
 kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights* w,
                                   const kvb_rope_table* rope,
                                   const float* x, const int32_t* row_idx,
                                   const int32_t* rope_pos, int64_t m,
                                   uint16_t* q_out, uint16_t* k_out, uint16_t* v_out,
-                                  const int32_t* kv_dst,
+                                  const int32_t* kv_dst, int64_t n_kv_rows,
                                   void* ws, size_t ws_bytes, void* stream);
 
 /* Allocation-free variant of kvb_gather_rmsnorm_qkv (the paper has no counterpart:
@@ -234,22 +277,25 @@ kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights
  * so the scratch this step needs (the m normalised bf16 rows that feed the GEMM)
  * lives in a fixed array inside the library, KVB_NOALLOC_MAX_ELEMS bf16 values
  * (8 MiB) that every GPU loading the library holds until the process exits.
- * Arguments and results are those of kvb_gather_rmsnorm_qkv without the workspace;
- * status_out (DEVICE int32, zeroed by the caller, or NULL) receives KVB_ERR_TIMEOUT
- * if a bounded wait in the GEMM runs out.  m * hidden above KVB_NOALLOC_MAX_ELEMS is
- * rejected with INVALID_ARG.  No memory is allocated or freed.  The first call on a
- * device looks the array's address up (cudaGetSymbolAddress) for that device, so make
- * it before any stream capture.  Every call reuses the same array (nothing in it has
- * to start at zero: each call overwrites the rows it reads); calls whose kernels
- * overlap on the GPU, e.g. on unordered streams, race on it.  Errors: INVALID_ARG,
- * UNSUPPORTED, CUDA. */
+ * Arguments, validation and results are those of kvb_gather_rmsnorm_qkv without the
+ * workspace; status_out (DEVICE int32, zeroed by the caller, or NULL) receives what the
+ * workspace status word would: KVB_ERR_TIMEOUT if a bounded wait in the GEMM runs out,
+ * KVB_ERR_INVALID_ARG for an index outside its range.  m * hidden above
+ * KVB_NOALLOC_MAX_ELEMS is rejected with INVALID_ARG.  No memory is allocated or freed.
+ * The first call on a device looks the array's address up (cudaGetSymbolAddress) for that
+ * device, so make it before any stream capture; the address is kept for the life of the
+ * process, so do not use this entry point on a device after cudaDeviceReset() there.
+ * Every call reuses the same array (nothing in it has to start at zero: each call
+ * overwrites the rows it reads); calls whose kernels overlap on the GPU, e.g. on
+ * unordered streams, race on it.  Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
 #define KVB_NOALLOC_MAX_ELEMS (4 * 1024 * 1024)
 kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, const kvb_layer_weights* w,
                                           const kvb_rope_table* rope,
                                           const float* x, const int32_t* row_idx,
                                           const int32_t* rope_pos, int64_t m,
                                           uint16_t* q_out, uint16_t* k_out, uint16_t* v_out,
-                                          const int32_t* kv_dst, int32_t* status_out, void* stream);
+                                          const int32_t* kv_dst, int64_t n_kv_rows,
+                                          int32_t* status_out, void* stream);
 
 /* KV scatter (Sec. 3.4: recomputed entries replace the cached ones): for r < m,
  *   k_dst[dst_idx[r]] = k_rows[r], v_dst[dst_idx[r]] = v_rows[r]   (kv_dim elements)
@@ -296,8 +342,9 @@ kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* byt
  *  4. layers >= check_layer: rows S = selected context rows + the n_query query rows,
  *     K/V scattered into the cache before attention over the whole cache;
  *  5. final RMSNorm of the query rows -> final_hidden [n_query][H] fp32.
- * k_chunks/v_chunks: [n_layers][n_ctx][Hkv][D] (K bf16, V fp16), each chunk's cache at
- * chunk-local positions (read only).  cache: output blended cache with n_rows >= n_ctx + n_query.
+ * k_chunks/v_chunks: chunk caches [n_layers][n_ctx][Hkv][D] (K and V bf16), each chunk's
+ * cache at chunk-local positions (read only).  cache: output blended cache (K bf16, V fp16)
+ * with n_rows >= n_ctx + n_query.
  * token_ids: DEVICE int32 [n_ctx + n_query]; chunk_start: DEVICE int32 [n_chunks+1]
  * with chunk_start[n_chunks] == n_ctx.  r in [0, 1]; 1 <= check_layer <= n_layers
  * (check_layer == n_layers means every layer is dense).  forced_sel: DEVICE int32
@@ -305,10 +352,12 @@ kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* byt
  * or NULL (receives the k chosen indices).  t: HOST timings or NULL (timing adds
  * events but no synchronisation until the call returns; with t != NULL the call
  * synchronises the stream once at the end to read the events).  r == 1 computes
- * the dense prefill of every layer.  Device-side checks: a token id outside [0, vocab)
- * embeds as a zero row and a forced_sel entry outside [0, n_ctx) is replaced by row 0;
- * both record KVB_ERR_INVALID_ARG in the workspace status word (kvb_device_status), and
- * the results of such a call are not meaningful.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
+ * the dense prefill of every layer.  taps: residual rows captured at layer boundaries
+ * (kvb_layer_taps), or NULL.  Device-side checks: a token id outside [0, vocab) embeds
+ * as a zero row and a forced_sel entry outside [0, n_ctx) is replaced by row 0; both
+ * record KVB_ERR_INVALID_ARG in the workspace status word (kvb_device_status), and a V
+ * value of the chunk caches outside fp16's range records KVB_ERR_RANGE; the results of
+ * such a call are not meaningful.  Errors: INVALID_ARG, WORKSPACE, CUDA. */
 kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
                                  const kvb_rope_table* rope,
                                  const uint16_t* k_chunks, const uint16_t* v_chunks,
@@ -318,7 +367,8 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
                                  float r, int32_t check_layer,
                                  const int32_t* forced_sel, int64_t forced_k,
                                  float* final_hidden, int32_t* sel_out,
-                                 kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
+                                 kvb_timings* t, const kvb_layer_taps* taps,
+                                 void* ws, size_t ws_bytes, void* stream);
 
 /* The same prefill with the chunk caches in pinned HOST memory, ingested layer by layer
  * while the model computes (Sec. 3.4: KV caches are transferred to the GPU, merged and
@@ -328,7 +378,7 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model,
  * `cache` there, and makes `stream` wait for that layer only just before it first reads
  * or writes cache layer l; layer 0 (and every layer before check_layer) needs no cache, so
  * the ingest runs under its compute.  k_chunks_host / v_chunks_host: pinned host memory
- * (cudaHostAlloc or registered), [n_layers][n_ctx][Hkv][D], K bf16 / V fp16.  copy_stream:
+ * (cudaHostAlloc or registered), [n_layers][n_ctx][Hkv][D], K and V bf16.  copy_stream:
  * a stream other than `stream`.  Workspace: kvb_workspace_size_pipelined(cfg, n_ctx +
  * n_query, n_ctx) bytes (the staging slots follow the regular layout).  All other
  * arguments and results as kvb_selective_prefill; realign_ms in `t` is 0 here because the
@@ -343,7 +393,8 @@ kvb_status kvb_selective_prefill_host(const kvb_config* cfg, const kvb_model* mo
                                       float r, int32_t check_layer,
                                       const int32_t* forced_sel, int64_t forced_k,
                                       float* final_hidden, int32_t* sel_out,
-                                      kvb_timings* t, void* ws, size_t ws_bytes,
+                                      kvb_timings* t, const kvb_layer_taps* taps,
+                                      void* ws, size_t ws_bytes,
                                       void* stream, void* copy_stream);
 
 /* Workspace bytes for kvb_selective_prefill_host: kvb_workspace_size(cfg, n_rows) plus two
@@ -355,16 +406,21 @@ kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, i
  *   row t attends cache rows [kv_lo[t], t] (kv_lo NULL = 0) with RoPE at rope_pos[t]
  *   (NULL = t).  With kv_lo = chunk start and rope_pos = t - chunk start every chunk
  *   is prefilled alone at chunk-local positions.
- * Writes every layer's K/V into cache rows [0, n) and, if final_hidden != NULL, the
- * final RMSNorm of the last n_out rows to final_hidden [n_out][H].  Token ids outside
- * [0, vocab) are reported in the status word as for kvb_selective_prefill.  Errors as
- * above. */
+ * Writes every layer's K/V into the blended-format cache rows [0, n) and, if
+ * v_chunk_out != NULL, every layer's V also in bf16 to v_chunk_out [n_layers][n][Hkv][D]
+ * (so that cache->k (with n_rows == n) and v_chunk_out form a chunk cache in the format
+ * kvb_selective_prefill reads).  If final_hidden != NULL, the final RMSNorm of the last
+ * n_out rows goes to final_hidden [n_out][H].  taps: as for kvb_selective_prefill (every
+ * layer is dense here), or NULL.  Token ids outside [0, vocab) are reported in the status
+ * word as for kvb_selective_prefill.  Errors as above. */
 kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model,
                             const kvb_rope_table* rope, kvb_kv_cache* cache,
+                            uint16_t* v_chunk_out,
                             const int32_t* token_ids, int64_t n,
                             const int32_t* rope_pos, const int32_t* kv_lo,
                             float* final_hidden, int64_t n_out,
-                            kvb_timings* t, void* ws, size_t ws_bytes, void* stream);
+                            kvb_timings* t, const kvb_layer_taps* taps,
+                            void* ws, size_t ws_bytes, void* stream);
 
 /* First token (the "first token" that closes time-to-first-token, Sec. 4.3): for n rows
  * of final hidden states h (fp32 [n][H], already through the final RMSNorm),
@@ -446,8 +502,9 @@ kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const 
                                 uint16_t* out, void* ws, size_t ws_bytes, void* stream);
 
 /* Synchronise `stream`, then read and clear the device status word that kernels using
- * workspace `ws` write when a bounded wait runs out.  *code_out receives KVB_OK or
- * KVB_ERR_TIMEOUT.  Errors: INVALID_ARG, CUDA. */
+ * workspace `ws` write when a bounded wait runs out or an index or value is out of range.
+ * *code_out receives KVB_OK or the first device-side error code recorded
+ * (KVB_ERR_TIMEOUT, KVB_ERR_INVALID_ARG, KVB_ERR_RANGE).  Errors: INVALID_ARG, CUDA. */
 kvb_status kvb_device_status(void* ws, size_t ws_bytes, void* stream, int32_t* code_out);
 
 /* Exercise the bounded-wait path (for tests; the paper has no counterpart): launch one

@@ -26,6 +26,8 @@ kvb_status fail(kvb_status s, const char* fmt, ...) {
     return s;
 }
 
+void clear_last_error() { g_err[0] = 0; }
+
 kvb_status cuda_ok(cudaError_t e, const char* what) {
     if (e == cudaSuccess) return KVB_OK;
     return fail(KVB_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
@@ -135,13 +137,7 @@ size_t workspace_layout(const kvb_config* c, int64_t n, void* base, Workspace* w
     return off;
 }
 
-}  // namespace kvb
-
-using namespace kvb;
-
-// ============================================================================ helpers
-
-static kvb_status check_cfg(const kvb_config* c) {
+kvb_status check_cfg(const kvb_config* c) {
     if (!c) return fail(KVB_ERR_INVALID_ARG, "config is NULL");
     if (c->hidden <= 0 || c->n_q_heads <= 0 || c->n_kv_heads <= 0 || c->head_dim <= 0 || c->mlp_dim <= 0 ||
         c->n_layers <= 0)
@@ -166,26 +162,13 @@ static kvb_status check_cfg(const kvb_config* c) {
     return KVB_OK;
 }
 
-// q.k multiplier of the softmax, times log2(e) (the kernels exponentiate base 2)
-static double attn_scale(const kvb_config* c) {
-    double s = 1.0 / sqrt((double)c->head_dim);
-    if (c->rope_scaling == KVB_ROPE_YARN) {
-        const double m = 0.1 * log((double)c->rs_factor) + 1.0;   // YaRN: sqrt(1/t)
-        s *= m * m;
-    }
-    return s;
-}
-static float attn_scale_log2(const kvb_config* c) {
-    return (float)(1.4426950408889634 * attn_scale(c));
-}
-
-static kvb_status check_ptr(const void* p, const char* name) {
+kvb_status check_ptr(const void* p, const char* name) {
     if (!p) return fail(KVB_ERR_INVALID_ARG, "%s is NULL", name);
     if (!aligned16(p)) return fail(KVB_ERR_INVALID_ARG, "%s is not 16-byte aligned", name);
     return KVB_OK;
 }
 
-static kvb_status check_layer(const kvb_layer_weights* w) {
+kvb_status check_weights(const kvb_layer_weights* w) {
     if (!w) return fail(KVB_ERR_INVALID_ARG, "layer weights are NULL");
     kvb_status s;
     if ((s = check_ptr(w->attn_norm, "attn_norm")) || (s = check_ptr(w->w_qkv, "w_qkv")) ||
@@ -197,7 +180,7 @@ static kvb_status check_layer(const kvb_layer_weights* w) {
     return KVB_OK;
 }
 
-static kvb_status check_rope(const kvb_rope_table* r, int64_t need_pos) {
+kvb_status check_rope(const kvb_rope_table* r, int64_t need_pos) {
     if (!r) return fail(KVB_ERR_INVALID_ARG, "rope table is NULL");
     kvb_status s;
     if ((s = check_ptr(r->cos, "rope cos")) || (s = check_ptr(r->sin, "rope sin"))) return s;
@@ -205,6 +188,25 @@ static kvb_status check_rope(const kvb_rope_table* r, int64_t need_pos) {
         return fail(KVB_ERR_INVALID_ARG, "rope table covers %lld positions, %lld needed", (long long)r->max_pos,
                     (long long)need_pos);
     return KVB_OK;
+}
+
+}  // namespace kvb
+
+using namespace kvb;
+
+// ============================================================================ helpers
+
+// q.k multiplier of the softmax, times log2(e) (the kernels exponentiate base 2)
+static double attn_scale(const kvb_config* c) {
+    double s = 1.0 / sqrt((double)c->head_dim);
+    if (c->rope_scaling == KVB_ROPE_YARN) {
+        const double m = 0.1 * log((double)c->rs_factor) + 1.0;   // YaRN: sqrt(1/t)
+        s *= m * m;
+    }
+    return s;
+}
+static float attn_scale_log2(const kvb_config* c) {
+    return (float)(1.4426950408889634 * attn_scale(c));
 }
 
 #define KVB_TRY(expr)                    \
@@ -302,14 +304,16 @@ Ctx make_ctx(const kvb_config* c, const kvb_rope_table* rope, const Workspace& w
     return x;
 }
 
-// a = RMSNorm(x[idx]) ; q, k, v = a W^T with RoPE
+// a = RMSNorm(x[idx]) ; q, k, v = a W^T with RoPE; k / v rows kv_dst[r] (or r) < n_kv_rows
 kvb_status qkv_rows(const Ctx& x, const kvb_layer_weights* lw, const float* xin, const int32_t* idx,
-                    const int32_t* rope_pos, int64_t m, uint16_t* q, uint16_t* k, uint16_t* v, const int32_t* kv_dst) {
+                    const int32_t* rope_pos, int64_t m, uint16_t* q, uint16_t* k, uint16_t* v, const int32_t* kv_dst,
+                    int64_t n_kv_rows, uint16_t* v_bf16 = nullptr) {
     KVB_TRY(launch_rmsnorm(xin, idx, m, x.H, lw->attn_norm, x.c->rms_eps, x.w.a, nullptr, x.st));
     GemmParams p{};
     p.M = m; p.N = x.QD + 2 * x.KVD; p.K = x.H; p.epi = EPI_QKV;
     p.col_base = 0; p.q_dim = x.QD; p.kv_dim = x.KVD; p.head_dim = x.D;
-    p.q_out = q; p.k_out = k; p.v_out = v; p.kv_dst = kv_dst; p.rope_pos = rope_pos;
+    p.q_out = q; p.k_out = k; p.v_out = v; p.kv_dst = kv_dst; p.n_kv_rows = n_kv_rows; p.v_out_bf16 = v_bf16;
+    p.rope_pos = rope_pos; p.max_pos = x.rope->max_pos;
     p.cos_t = x.rope->cos; p.sin_t = x.rope->sin; p.bias = lw->b_qkv; p.status = x.w.status;
     return gemm(x, p, x.w.a, x.H, lw->w_qkv, x.H, nullptr);
 }
@@ -342,10 +346,12 @@ kvb_status attn_rows(const Ctx& x, const uint16_t* q, const int32_t* q_idx, cons
 }
 
 // one decoder layer over m rows whose residual is the dense buffer xio [m][H]
-//   row r: cache row kv_row[r] (NULL: r), RoPE position rope_pos[r], keys [kv_lo[r], kv_row[r]]
+//   row r: cache row kv_row[r] (NULL: r), RoPE position rope_pos[r], keys [kv_lo[r], kv_row[r]];
+//   v_bf16: optional bf16 copy of the layer's V rows (chunk-cache format)
 kvb_status layer(const Ctx& x, const kvb_layer_weights* lw, float* xio, int64_t m, const int32_t* kv_row,
-                 const int32_t* rope_pos, const int32_t* kv_lo, uint16_t* kc, uint16_t* vc, int64_t n_kv) {
-    KVB_TRY(qkv_rows(x, lw, xio, nullptr, rope_pos, m, x.w.q, kc, vc, kv_row));
+                 const int32_t* rope_pos, const int32_t* kv_lo, uint16_t* kc, uint16_t* vc, int64_t n_kv,
+                 uint16_t* v_bf16 = nullptr) {
+    KVB_TRY(qkv_rows(x, lw, xio, nullptr, rope_pos, m, x.w.q, kc, vc, kv_row, n_kv, v_bf16));
     KVB_TRY(attn_rows(x, x.w.q, kv_row ? kv_row : x.w.ident, kv_lo, m, kc, vc, n_kv, x.w.attn, kv_row != nullptr));
     return mlp_rows(x, lw, x.w.attn, m, xio);
 }
@@ -375,6 +381,41 @@ struct Timer {
     }
 };
 
+// Layer-boundary captures of the residual rows (kvb_layer_taps).
+struct Taps {
+    const kvb_layer_taps* t = nullptr;
+    int H = 0;
+    cudaStream_t st = nullptr;
+    // copy `rows` residual rows entering layer l (n_layers: leaving the last one) into every slot asking for l
+    kvb_status at(int l, const float* x, int64_t rows) const {
+        if (!t) return KVB_OK;
+        for (int i = 0; i < t->n; ++i) {
+            if (t->layers[i] != l) continue;
+            KVB_TRY(cuda_ok(cudaMemcpyAsync(t->x_out + (size_t)i * t->rows_cap * H, x, (size_t)rows * H * 4,
+                                            cudaMemcpyDeviceToDevice, st), "layer tap copy"));
+            if (t->rows_out) t->rows_out[i] = rows;
+        }
+        return KVB_OK;
+    }
+};
+
+// Validates taps against the rows each boundary carries: layers below `first_sel` (and the
+// end, when first_sel == n_layers) carry n_dense rows, the others n_sel.
+kvb_status check_taps(const kvb_layer_taps* t, int n_layers, int first_sel, int64_t n_dense, int64_t n_sel) {
+    if (!t || t->n == 0) return KVB_OK;
+    if (t->n < 0 || !t->layers || t->rows_cap < 0) return fail(KVB_ERR_INVALID_ARG, "taps: bad count, layers or rows_cap");
+    KVB_TRY(check_ptr(t->x_out, "taps x_out"));
+    for (int i = 0; i < t->n; ++i) {
+        const int l = t->layers[i];
+        if (l < 0 || l > n_layers) return fail(KVB_ERR_INVALID_ARG, "taps: layer %d not in [0, %d]", l, n_layers);
+        const int64_t need = (l < first_sel || first_sel >= n_layers) ? n_dense : n_sel;
+        if (need > t->rows_cap)
+            return fail(KVB_ERR_INVALID_ARG, "taps: layer %d carries %lld rows, rows_cap is %lld", l,
+                        (long long)need, (long long)t->rows_cap);
+    }
+    return KVB_OK;
+}
+
 }  // namespace
 
 static void fill_kernel_times(const Prof& prof, kvb_timings* t, int64_t launches) {
@@ -403,16 +444,17 @@ const char* kvb_status_string(kvb_status s) {
         case KVB_ERR_CUDA: return "CUDA error";
         case KVB_ERR_TIMEOUT: return "device wait timed out";
         case KVB_ERR_WORKSPACE: return "workspace too small";
+        case KVB_ERR_RANGE: return "value out of range";
         default: return "unknown status";
     }
 }
 
 const char* kvb_last_error(void) { return g_err; }
 
-int32_t kvb_version(void) { return 200; }
+int32_t kvb_version(void) { return 300; }
 
 kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos, float* cos_host, float* sin_host) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (max_pos < 1 || !cos_host || !sin_host) return fail(KVB_ERR_INVALID_ARG, "rope table: bad size or pointer");
     const int half = cfg->head_dim / 2;
@@ -428,7 +470,7 @@ kvb_status kvb_rope_table_fill(const kvb_config* cfg, int64_t max_pos, float* co
 }
 
 kvb_status kvb_attention_scale(const kvb_config* cfg, float* scale_out) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (!scale_out) return fail(KVB_ERR_INVALID_ARG, "attention scale: NULL output");
     *scale_out = (float)attn_scale(cfg);
@@ -438,8 +480,8 @@ kvb_status kvb_attention_scale(const kvb_config* cfg, float* scale_out) {
 kvb_status kvb_rope_realign(const kvb_config* cfg, const kvb_rope_table* rope, const uint16_t* k_src,
                             const uint16_t* v_src, int64_t src_rows, uint16_t* k_dst, uint16_t* v_dst,
                             int64_t dst_rows, int32_t layer_begin, int32_t layer_end, const int32_t* chunk_start,
-                            int32_t n_chunks, int64_t n_ctx, void* stream) {
-    g_err[0] = 0;
+                            int32_t n_chunks, int64_t n_ctx, void* ws, size_t ws_bytes, void* stream) {
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (layer_begin < 0 || layer_end < layer_begin || layer_end > cfg->n_layers)
         return fail(KVB_ERR_INVALID_ARG, "realign: bad layer range [%d, %d)", layer_begin, layer_end);
@@ -450,18 +492,22 @@ kvb_status kvb_rope_realign(const kvb_config* cfg, const kvb_rope_table* rope, c
     KVB_TRY(check_ptr(k_src, "k_src"));
     KVB_TRY(check_ptr(k_dst, "k_dst"));
     KVB_TRY(check_ptr(chunk_start, "chunk_start"));
-    if (v_src && v_dst && v_src != v_dst) {
+    const bool with_v = v_src && v_dst;
+    if (with_v) {
         KVB_TRY(check_ptr(v_src, "v_src"));
         KVB_TRY(check_ptr(v_dst, "v_dst"));
+        if (!ws || ws_bytes < 256) return fail(KVB_ERR_WORKSPACE, "realign: V conversion needs a 256-byte status workspace");
     }
-    if (k_src == k_dst && src_rows != dst_rows) return fail(KVB_ERR_INVALID_ARG, "realign: in place needs equal strides");
+    if ((k_src == k_dst || (with_v && v_src == v_dst)) && src_rows != dst_rows)
+        return fail(KVB_ERR_INVALID_ARG, "realign: in place needs equal strides");
     KVB_TRY(check_rope(rope, n_ctx));
     const int64_t kvd = (int64_t)cfg->n_kv_heads * cfg->head_dim;
     const int64_t lb = layer_begin;
     return launch_realign(rope->cos, rope->sin, cfg->head_dim, cfg->n_kv_heads, k_src + lb * src_rows * kvd,
-                          v_src ? v_src + lb * src_rows * kvd : nullptr, src_rows * kvd, k_dst + lb * dst_rows * kvd,
-                          v_dst ? v_dst + lb * dst_rows * kvd : nullptr, dst_rows * kvd, layer_end - layer_begin,
-                          chunk_start, n_chunks, n_ctx, static_cast<cudaStream_t>(stream));
+                          with_v ? v_src + lb * src_rows * kvd : nullptr, src_rows * kvd, k_dst + lb * dst_rows * kvd,
+                          with_v ? v_dst + lb * dst_rows * kvd : nullptr, dst_rows * kvd, layer_end - layer_begin,
+                          chunk_start, n_chunks, n_ctx, with_v ? static_cast<int*>(ws) : nullptr,
+                          static_cast<cudaStream_t>(stream));
 }
 
 size_t kvb_hkvd_workspace_size(int64_t n_ctx) { return hkvd_ws_bytes(n_ctx); }
@@ -469,7 +515,7 @@ size_t kvb_hkvd_workspace_size(int64_t n_ctx) { return hkvd_ws_bytes(n_ctx); }
 kvb_status kvb_hkvd_select(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t* k_cached, int64_t ld_cached,
                            int64_t n_ctx, int32_t kv_dim, int64_t k, int32_t* sel_out, float* dev_out, void* ws,
                            size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     if (n_ctx < 0 || k < 0 || k > n_ctx) return fail(KVB_ERR_INVALID_ARG, "hkvd: need 0 <= k <= n_ctx");
     if (kv_dim <= 0 || kv_dim % 8 || ld_fresh < kv_dim || ld_cached < kv_dim || ld_fresh % 8 || ld_cached % 8)
         return fail(KVB_ERR_INVALID_ARG, "hkvd: kv_dim and leading dims must be multiples of 8");
@@ -486,7 +532,7 @@ kvb_status kvb_hkvd_select(const uint16_t* k_fresh, int64_t ld_fresh, const uint
 }
 
 kvb_status kvb_workspace_size(const kvb_config* cfg, int64_t n_rows, size_t* bytes) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (!bytes || n_rows < 0) return fail(KVB_ERR_INVALID_ARG, "workspace size: bad arguments");
     Workspace w;
@@ -504,12 +550,12 @@ static kvb_status carve(const kvb_config* cfg, int64_t n, void* ws, size_t ws_by
 
 kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights* w, const kvb_rope_table* rope,
                                   const float* x, const int32_t* row_idx, const int32_t* rope_pos, int64_t m,
-                                  uint16_t* q_out, uint16_t* k_out, uint16_t* v_out, const int32_t* kv_dst, void* ws,
-                                  size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+                                  uint16_t* q_out, uint16_t* k_out, uint16_t* v_out, const int32_t* kv_dst,
+                                  int64_t n_kv_rows, void* ws, size_t ws_bytes, void* stream) {
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
-    KVB_TRY(check_layer(w));
-    if (m < 0) return fail(KVB_ERR_INVALID_ARG, "m < 0");
+    KVB_TRY(check_weights(w));
+    if (m < 0 || n_kv_rows < 0) return fail(KVB_ERR_INVALID_ARG, "m < 0 or n_kv_rows < 0");
     if (m == 0) return KVB_OK;
     KVB_TRY(check_ptr(x, "x"));
     KVB_TRY(check_ptr(rope_pos, "rope_pos"));
@@ -520,12 +566,12 @@ kvb_status kvb_gather_rmsnorm_qkv(const kvb_config* cfg, const kvb_layer_weights
     Workspace wsl;
     KVB_TRY(carve(cfg, m, ws, ws_bytes, &wsl));
     Ctx c = make_ctx(cfg, rope, wsl, stream);
-    return qkv_rows(c, w, x, row_idx, rope_pos, m, q_out, k_out, v_out, kv_dst);
+    return qkv_rows(c, w, x, row_idx, rope_pos, m, q_out, k_out, v_out, kv_dst, n_kv_rows);
 }
 
 kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const int32_t* dst_idx, int64_t m,
                           int32_t kv_dim, uint16_t* k_dst, uint16_t* v_dst, int64_t n_dst_rows, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     if (m < 0 || kv_dim <= 0 || kv_dim % 8 || m > n_dst_rows)
         return fail(KVB_ERR_INVALID_ARG, "scatter: bad sizes (m %lld, kv_dim %d, rows %lld)", (long long)m, kv_dim,
                     (long long)n_dst_rows);
@@ -542,7 +588,7 @@ kvb_status kvb_kv_scatter(const uint16_t* k_rows, const uint16_t* v_rows, const 
 kvb_status kvb_sparse_query_attn(const kvb_config* cfg, const uint16_t* q, const int32_t* q_idx,
                                  const int32_t* kv_lo, int64_t m, const uint16_t* k_cache, const uint16_t* v_cache,
                                  int64_t n_kv, uint16_t* out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (m < 0 || n_kv < 1 || n_kv > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "attention: bad sizes");
     if (m == 0) return KVB_OK;
@@ -560,9 +606,9 @@ kvb_status kvb_sparse_query_attn(const kvb_config* cfg, const uint16_t* q, const
 
 kvb_status kvb_mlp_rows(const kvb_config* cfg, const kvb_layer_weights* w, const uint16_t* attn, int64_t m, float* x,
                         void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
-    KVB_TRY(check_layer(w));
+    KVB_TRY(check_weights(w));
     if (m < 0) return fail(KVB_ERR_INVALID_ARG, "m < 0");
     if (m == 0) return KVB_OK;
     KVB_TRY(check_ptr(attn, "attn"));
@@ -577,7 +623,7 @@ static kvb_status check_model(const kvb_config* cfg, const kvb_model* model) {
     if (!model || !model->layers) return fail(KVB_ERR_INVALID_ARG, "model or its layer array is NULL");
     KVB_TRY(check_ptr(model->embed, "embed"));
     KVB_TRY(check_ptr(model->final_norm, "final_norm"));
-    for (int l = 0; l < cfg->n_layers; ++l) KVB_TRY(check_layer(&model->layers[l]));
+    for (int l = 0; l < cfg->n_layers; ++l) KVB_TRY(check_weights(&model->layers[l]));
     return KVB_OK;
 }
 
@@ -592,10 +638,10 @@ static kvb_status check_cache(const kvb_config* cfg, const kvb_kv_cache* cache, 
 }
 
 kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
-                            kvb_kv_cache* cache, const int32_t* token_ids, int64_t n, const int32_t* rope_pos,
-                            const int32_t* kv_lo, float* final_hidden, int64_t n_out, kvb_timings* t, void* ws,
-                            size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+                            kvb_kv_cache* cache, uint16_t* v_chunk_out, const int32_t* token_ids, int64_t n,
+                            const int32_t* rope_pos, const int32_t* kv_lo, float* final_hidden, int64_t n_out,
+                            kvb_timings* t, const kvb_layer_taps* taps, void* ws, size_t ws_bytes, void* stream) {
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     KVB_TRY(check_model(cfg, model));
     if (n < 1 || n > 0x7FFFFFFF || n_out < 0 || n_out > n) return fail(KVB_ERR_INVALID_ARG, "full prefill: bad n/n_out");
@@ -603,9 +649,13 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
     KVB_TRY(check_ptr(token_ids, "token_ids"));
     KVB_TRY(check_rope(rope, rope_pos ? 1 : n));
     if (final_hidden && n_out > 0) KVB_TRY(check_ptr(final_hidden, "final_hidden"));
+    if (v_chunk_out) KVB_TRY(check_ptr(v_chunk_out, "v_chunk_out"));
+    KVB_TRY(check_taps(taps, cfg->n_layers, cfg->n_layers, n, n));
     Workspace w;
     KVB_TRY(carve(cfg, n, ws, ws_bytes, &w));
     Ctx c = make_ctx(cfg, rope, w, stream);
+    Taps tap;
+    tap.t = taps; tap.H = c.H; tap.st = c.st;
     Prof prof;
     prof.st = c.st;
     if (t) c.prof = &prof;
@@ -618,8 +668,11 @@ kvb_status kvb_full_prefill(const kvb_config* cfg, const kvb_model* model, const
     for (int l = 0; l < cfg->n_layers; ++l) {
         uint16_t* kc = cache->k + (int64_t)l * cache->n_rows * kvd;
         uint16_t* vc = cache->v + (int64_t)l * cache->n_rows * kvd;
-        KVB_TRY(layer(c, &model->layers[l], w.x_all, n, nullptr, rope_pos ? rope_pos : w.ident, kv_lo, kc, vc, n));
+        KVB_TRY(tap.at(l, w.x_all, n));
+        KVB_TRY(layer(c, &model->layers[l], w.x_all, n, nullptr, rope_pos ? rope_pos : w.ident, kv_lo, kc, vc, n,
+                      v_chunk_out ? v_chunk_out + (int64_t)l * n * kvd : nullptr));
     }
+    KVB_TRY(tap.at(cfg->n_layers, w.x_all, n));
     tm.mark();
     if (final_hidden && n_out > 0)
         KVB_TRY(launch_rmsnorm(w.x_all + (n - n_out) * c.H, nullptr, n_out, c.H, model->final_norm, cfg->rms_eps,
@@ -655,9 +708,10 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
                                  const uint16_t* k_chunks, const uint16_t* v_chunks, kvb_kv_cache* cache,
                                  const int32_t* token_ids, const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
                                  int64_t n_query, float r, int32_t check_layer_idx, const int32_t* forced_sel,
-                                 int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
-                                 size_t ws_bytes, void* stream, bool host_src, void* copy_stream) {
-    g_err[0] = 0;
+                                 int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t,
+                                 const kvb_layer_taps* taps, void* ws, size_t ws_bytes, void* stream, bool host_src,
+                                 void* copy_stream) {
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     KVB_TRY(check_model(cfg, model));
     const int L = cfg->n_layers;
@@ -676,6 +730,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
     int64_t k = (int64_t)floor((double)r * (double)n_ctx + 1e-9);
     if (forced_sel) k = forced_k;
     const bool dense_all = check_layer_idx >= L || (!forced_sel && k >= n_ctx);
+    KVB_TRY(check_taps(taps, L, dense_all ? L : check_layer_idx, N, k + n_query));
     if (!dense_all && n_ctx > 0) {
         KVB_TRY(check_ptr(k_chunks, "k_chunks"));
         KVB_TRY(check_ptr(v_chunks, "v_chunks"));
@@ -698,6 +753,8 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
         return fail(KVB_ERR_WORKSPACE, "workspace %zu bytes < %zu needed", ws_bytes, ws_need);
     KVB_TRY(carve(cfg, N, ws, ws_bytes, &w));
     Ctx c = make_ctx(cfg, rope, w, stream);
+    Taps tap;
+    tap.t = taps; tap.H = c.H; tap.st = c.st;
     Prof prof;
     prof.st = c.st;
     if (t) c.prof = &prof;
@@ -721,7 +778,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
     if (lc < L && n_ctx > 0 && !host_src) {
         KVB_TRY(launch_realign(rope->cos, rope->sin, c.D, c.Hkv, k_chunks + (int64_t)lc * n_ctx * kvd,
                                v_chunks + (int64_t)lc * n_ctx * kvd, n_ctx * kvd, kc(lc), vc(lc), rows_c * kvd,
-                               L - lc, chunk_start, n_chunks, n_ctx, c.st));
+                               L - lc, chunk_start, n_chunks, n_ctx, w.status, c.st));
     } else if (lc < L && n_ctx > 0) {
         cudaStream_t cs = static_cast<cudaStream_t>(copy_stream);
         cudaEvent_t go = nullptr;
@@ -742,7 +799,7 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
             KVB_TRY(cuda_ok(cudaMemcpyAsync(sv, v_chunks + (size_t)l * layer_elems, layer_elems * 2,
                                             cudaMemcpyHostToDevice, cs), "pipelined prefill: V copy"));
             KVB_TRY(launch_realign(rope->cos, rope->sin, c.D, c.Hkv, sk, sv, (int64_t)layer_elems, kc(l), vc(l),
-                                   rows_c * kvd, 1, chunk_start, n_chunks, n_ctx, cs));
+                                   rows_c * kvd, 1, chunk_start, n_chunks, n_ctx, w.status, cs));
             KVB_TRY(cuda_ok(cudaEventCreateWithFlags(&ready.ev[l], cudaEventDisableTiming), "pipelined prefill: event"));
             KVB_TRY(cuda_ok(cudaEventRecord(ready.ev[l], cs), "pipelined prefill: record"));
         }
@@ -755,8 +812,10 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
     // 2. dense layers (layer 0 at least): every row, causal
     KVB_TRY(launch_iota(w.ident, N, 0, c.st));
     KVB_TRY(launch_embed(model->embed, token_ids, N, c.H, cfg->vocab, w.x_all, w.status, c.st));
-    for (int l = 0; l < lc; ++l)
+    for (int l = 0; l < lc; ++l) {
+        KVB_TRY(tap.at(l, w.x_all, N));
         KVB_TRY(layer(c, &model->layers[l], w.x_all, N, nullptr, w.ident, nullptr, kc(l), vc(l), N));
+    }
     tm.mark();
     float* x_final = w.x_all;
     int64_t m = N;
@@ -770,7 +829,8 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
                 GemmParams p{};
                 p.M = n_ctx; p.N = c.KVD; p.K = c.H; p.epi = EPI_QKV;
                 p.col_base = c.QD; p.q_dim = c.QD; p.kv_dim = c.KVD; p.head_dim = c.D;
-                p.k_out = w.k_fresh; p.rope_pos = w.ident; p.cos_t = rope->cos; p.sin_t = rope->sin;
+                p.k_out = w.k_fresh; p.n_kv_rows = n_ctx; p.rope_pos = w.ident; p.max_pos = rope->max_pos;
+                p.cos_t = rope->cos; p.sin_t = rope->sin;
                 p.bias = lw->b_qkv; p.status = w.status;
                 KVB_TRY(gemm(c, p, w.a, c.H, lw->w_qkv + (int64_t)c.QD * c.H, c.H, nullptr));
                 KVB_TRY(wait_layer(lc));
@@ -789,10 +849,13 @@ static kvb_status selective_impl(const kvb_config* cfg, const kvb_model* model, 
         // 4. selective layers over the recomputed rows
         for (int l = lc; l < L; ++l) {
             KVB_TRY(wait_layer(l));
+            KVB_TRY(tap.at(l, w.x_sel, m));
             KVB_TRY(layer(c, &model->layers[l], w.x_sel, m, w.rows, w.rows, nullptr, kc(l), vc(l), N));
         }
+        KVB_TRY(tap.at(L, w.x_sel, m));
         x_final = w.x_sel;
     } else {
+        KVB_TRY(tap.at(L, w.x_all, N));
         if (sel_out && n_ctx > 0) KVB_TRY(launch_iota(sel_out, n_ctx, 0, c.st));
         k = n_ctx;
         tm.mark();
@@ -826,10 +889,10 @@ kvb_status kvb_selective_prefill(const kvb_config* cfg, const kvb_model* model, 
                                  const uint16_t* k_chunks, const uint16_t* v_chunks, kvb_kv_cache* cache,
                                  const int32_t* token_ids, const int32_t* chunk_start, int32_t n_chunks, int64_t n_ctx,
                                  int64_t n_query, float r, int32_t check_layer, const int32_t* forced_sel,
-                                 int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
-                                 size_t ws_bytes, void* stream) {
+                                 int64_t forced_k, float* final_hidden, int32_t* sel_out, kvb_timings* t,
+                                 const kvb_layer_taps* taps, void* ws, size_t ws_bytes, void* stream) {
     return selective_impl(cfg, model, rope, k_chunks, v_chunks, cache, token_ids, chunk_start, n_chunks, n_ctx,
-                          n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, ws, ws_bytes,
+                          n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, taps, ws, ws_bytes,
                           stream, false, nullptr);
 }
 
@@ -838,16 +901,18 @@ kvb_status kvb_selective_prefill_host(const kvb_config* cfg, const kvb_model* mo
                                       kvb_kv_cache* cache, const int32_t* token_ids, const int32_t* chunk_start,
                                       int32_t n_chunks, int64_t n_ctx, int64_t n_query, float r,
                                       int32_t check_layer, const int32_t* forced_sel, int64_t forced_k,
-                                      float* final_hidden, int32_t* sel_out, kvb_timings* t, void* ws,
-                                      size_t ws_bytes, void* stream, void* copy_stream) {
+                                      float* final_hidden, int32_t* sel_out, kvb_timings* t,
+                                      const kvb_layer_taps* taps, void* ws, size_t ws_bytes, void* stream,
+                                      void* copy_stream) {
+    clear_last_error();
     if (copy_stream == stream) return fail(KVB_ERR_INVALID_ARG, "pipelined prefill: copy_stream must differ from stream");
     return selective_impl(cfg, model, rope, k_chunks_host, v_chunks_host, cache, token_ids, chunk_start, n_chunks,
-                          n_ctx, n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, ws, ws_bytes,
-                          stream, true, copy_stream);
+                          n_ctx, n_query, r, check_layer, forced_sel, forced_k, final_hidden, sel_out, t, taps, ws,
+                          ws_bytes, stream, true, copy_stream);
 }
 
 kvb_status kvb_workspace_size_pipelined(const kvb_config* cfg, int64_t n_rows, int64_t n_ctx, size_t* bytes) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (!bytes || n_rows < 0 || n_ctx < 0) return fail(KVB_ERR_INVALID_ARG, "workspace size: bad arguments");
     Workspace w;
@@ -867,7 +932,7 @@ size_t kvb_window_select_workspace_size(int64_t n_ctx) { return 256 + round16(n_
 
 kvb_status kvb_window_select(const int32_t* win_start, int32_t n_win, int32_t window, int64_t n_ctx, int32_t* sel_out,
                              int64_t* k_out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     if (n_win < 0 || window < 0 || n_ctx < 0 || n_ctx > 0x7FFFFFFF || (int64_t)n_win * window > 0x7FFFFFFF)
         return fail(KVB_ERR_INVALID_ARG, "window select: need 0 <= n_win, window; n_win * window and n_ctx < 2^31");
     if (n_win > 0) KVB_TRY(check_ptr4(win_start, "win_start"));
@@ -883,7 +948,7 @@ kvb_status kvb_window_select(const int32_t* win_start, int32_t n_win, int32_t wi
 kvb_status kvb_key_deviation_histogram(const uint16_t* k_a, int64_t ld_a, const uint16_t* k_b, int64_t ld_b, int64_t n,
                                        int32_t kv_dim, const float* edges, int32_t n_edges, float* dev_out,
                                        int64_t* hist_out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     if (n < 0 || n > 0x7FFFFFFF) return fail(KVB_ERR_INVALID_ARG, "deviation histogram: n out of range");
     if (kv_dim <= 0 || kv_dim % 8 || ld_a < kv_dim || ld_b < kv_dim || ld_a % 8 || ld_b % 8)
         return fail(KVB_ERR_INVALID_ARG, "deviation histogram: kv_dim and leading dims must be multiples of 8");
@@ -906,7 +971,7 @@ kvb_status kvb_key_deviation_histogram(const uint16_t* k_a, int64_t ld_a, const 
 
 kvb_status kvb_lm_head_argmax(const kvb_config* cfg, const uint16_t* lm_head, const float* hidden, int32_t n,
                               float* logits_out, int32_t* tokens_out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_cfg(cfg));
     if (n < 1 || n > KVB_LMHEAD_MAX_ROWS || cfg->vocab < 1 || cfg->hidden > 8192 || cfg->hidden % 8)
         return fail(KVB_ERR_INVALID_ARG, "lm head: need 1 <= n <= %d rows, vocab >= 1, hidden <= 8192",
@@ -968,7 +1033,7 @@ static kvb_status check_decode(const kvb_config* cfg, int64_t max_pos) {
 }
 
 kvb_status kvb_decode_workspace_size(const kvb_config* cfg, int64_t max_pos, size_t* bytes) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_decode(cfg, max_pos));
     if (!bytes) return fail(KVB_ERR_INVALID_ARG, "decode workspace size: bytes is NULL");
     DecodeWs w;
@@ -979,7 +1044,7 @@ kvb_status kvb_decode_workspace_size(const kvb_config* cfg, int64_t max_pos, siz
 kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const uint16_t* k_layer,
                                 const uint16_t* v_layer, int64_t n_rows, const int32_t* pos, int64_t max_pos,
                                 uint16_t* out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_decode(cfg, max_pos));
     if (n_rows < max_pos) return fail(KVB_ERR_INVALID_ARG, "decode attention: n_rows %lld < max_pos %lld",
                                       (long long)n_rows, (long long)max_pos);
@@ -1000,7 +1065,7 @@ kvb_status kvb_decode_attention(const kvb_config* cfg, const uint16_t* q, const 
 kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const kvb_rope_table* rope,
                            const kvb_kv_cache* cache, const uint16_t* lm_head, int32_t* tokens, int32_t* pos,
                            int64_t max_pos, float* hidden_out, void* ws, size_t ws_bytes, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     KVB_TRY(check_decode(cfg, max_pos));
     if (cfg->vocab < 1 || cfg->hidden > 8192) return fail(KVB_ERR_UNSUPPORTED, "decode: vocab >= 1, hidden <= 8192");
     KVB_TRY(check_model(cfg, model));
@@ -1054,14 +1119,14 @@ kvb_status kvb_decode_step(const kvb_config* cfg, const kvb_model* model, const 
 }
 
 kvb_status kvb_debug_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
-    g_err[0] = 0;
+    clear_last_error();
     if (!ws || ws_bytes < 256 || limit_ns < 1000 || limit_ns > 4000000000ll)
         return fail(KVB_ERR_INVALID_ARG, "debug wait: bad workspace or limit");
     return launch_wait_timeout(static_cast<int*>(ws), (uint64_t)limit_ns, static_cast<cudaStream_t>(stream));
 }
 
 kvb_status kvb_device_status(void* ws, size_t ws_bytes, void* stream, int32_t* code_out) {
-    g_err[0] = 0;
+    clear_last_error();
     if (!ws || ws_bytes < 256 || !code_out) return fail(KVB_ERR_INVALID_ARG, "device status: bad arguments");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     KVB_TRY(cuda_ok(cudaStreamSynchronize(st), "device status sync"));

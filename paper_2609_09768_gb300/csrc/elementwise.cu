@@ -8,14 +8,32 @@ namespace kvb {
 namespace {
 
 // ------------------------------------------------------------------ re-alignment
+// bf16 pair (chunk-cache V) -> fp16 pair (blended-cache V container).  Exact for
+// 2^-14 <= |v| <= 65504 and 0 (a bf16 value has 8 significant bits, fp16 11); smaller
+// magnitudes round to fp16's subnormal spacing.  |v| > 65504 cannot be held: it is
+// written as +-65504 and `bad` is set; NaN stays NaN and also sets `bad`.
+KVB_DEV uint32_t v_bf16x2_to_f16x2(uint32_t v, bool& bad) {
+    const float a = bf16_lo(v), b = bf16_hi(v);
+    bad |= !(fabsf(a) <= 65504.f) || !(fabsf(b) <= 65504.f);
+    const float ca = (a != a) ? a : fminf(fmaxf(a, -65504.f), 65504.f);
+    const float cb = (b != b) ? b : fminf(fmaxf(b, -65504.f), 65504.f);
+    return pack_f16(ca, cb);
+}
+KVB_DEV uint4 v_convert16(uint4 u, bool& bad) {
+    return make_uint4(v_bf16x2_to_f16x2(u.x, bad), v_bf16x2_to_f16x2(u.y, bad), v_bf16x2_to_f16x2(u.z, bad),
+                      v_bf16x2_to_f16x2(u.w, bad));
+}
+
 // Thread item = (context row t, head h, group of 8 rotation pairs); the chunk
-// offset and its cos/sin are looked up once and reused for every layer.
+// offset and its cos/sin are looked up once and reused for every layer.  K is rotated
+// (bf16 in and out), V converted from bf16 to its fp16 container in the same pass.
 template <int D>
 __global__ void __launch_bounds__(256)
 realign_kernel(const float* __restrict__ cos_t, const float* __restrict__ sin_t, int Hkv,
-               const uint16_t* __restrict__ k_src, const uint16_t* __restrict__ v_src, int64_t src_ls,
-               uint16_t* __restrict__ k_dst, uint16_t* __restrict__ v_dst, int64_t dst_ls, int n_layers,
-               const int32_t* __restrict__ chunk_start, int n_chunks, int64_t n_ctx, bool copy_v) {
+               const uint16_t* k_src, const uint16_t* v_src, int64_t src_ls,   // may alias k_dst / v_dst
+               uint16_t* k_dst, uint16_t* v_dst, int64_t dst_ls, int n_layers,
+               const int32_t* __restrict__ chunk_start, int n_chunks, int64_t n_ctx, bool copy_v, int* status) {
+    bool bad = false;
     constexpr int GPH = D / 16;   // groups of 8 pairs per head
     const int64_t per_row = (int64_t)Hkv * GPH;
     const int64_t items = n_ctx * per_row;
@@ -71,13 +89,14 @@ realign_kernel(const float* __restrict__ cos_t, const float* __restrict__ sin_t,
                     __stcs(reinterpret_cast<uint4*>(k_dst + o), make_uint4(ra[0], ra[1], ra[2], ra[3]));
                     __stcs(reinterpret_cast<uint4*>(k_dst + o + D / 2), make_uint4(rb[0], rb[1], rb[2], rb[3]));
                     if (copy_v) {
-                        __stcs(reinterpret_cast<uint4*>(v_dst + o), va[u]);
-                        __stcs(reinterpret_cast<uint4*>(v_dst + o + D / 2), vb[u]);
+                        __stcs(reinterpret_cast<uint4*>(v_dst + o), v_convert16(va[u], bad));
+                        __stcs(reinterpret_cast<uint4*>(v_dst + o + D / 2), v_convert16(vb[u], bad));
                     }
                 }
             }
         }
     }
+    if (bad) set_status(status, KVB_ERR_RANGE);
 }
 
 // ------------------------------------------------------------------ embedding
@@ -211,17 +230,18 @@ unsigned grid_for(int64_t items, int threads) {
 
 kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv, const uint16_t* k_src,
                           const uint16_t* v_src, int64_t src_ls, uint16_t* k_dst, uint16_t* v_dst, int64_t dst_ls,
-                          int n_layers, const int32_t* chunk_start, int n_chunks, int64_t n_ctx, cudaStream_t st) {
+                          int n_layers, const int32_t* chunk_start, int n_chunks, int64_t n_ctx, int* status,
+                          cudaStream_t st) {
     if (n_layers <= 0 || n_ctx <= 0) return KVB_OK;
-    const bool copy_v = v_src && v_dst && v_src != v_dst;
+    const bool copy_v = v_src && v_dst;
     const int64_t items = n_ctx * Hkv * (D / 16);
     const unsigned grid = grid_for(items, 256);
     if (D == 128)
         realign_kernel<128><<<grid, 256, 0, st>>>(cos_t, sin_t, Hkv, k_src, v_src, src_ls, k_dst, v_dst, dst_ls,
-                                                  n_layers, chunk_start, n_chunks, n_ctx, copy_v);
+                                                  n_layers, chunk_start, n_chunks, n_ctx, copy_v, status);
     else if (D == 64)
         realign_kernel<64><<<grid, 256, 0, st>>>(cos_t, sin_t, Hkv, k_src, v_src, src_ls, k_dst, v_dst, dst_ls,
-                                                 n_layers, chunk_start, n_chunks, n_ctx, copy_v);
+                                                 n_layers, chunk_start, n_chunks, n_ctx, copy_v, status);
     else
         return fail(KVB_ERR_UNSUPPORTED, "realign: head_dim %d not built", D);
     count_launch();

@@ -190,25 +190,38 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
 
             if constexpr (EPI == EPI_QKV) {
                 constexpr int NH = BN / HD;
-                const int pos = valid ? p.rope_pos[row] : 0;
-                const float* crow = p.cos_t + (int64_t)pos * (HD / 2);
-                const float* srow = p.sin_t + (int64_t)pos * (HD / 2);
+                // indices the caller supplies are checked where they are used: a position outside the
+                // RoPE tables is rotated by position 0, a destination outside the k / v buffers writes
+                // nothing; both are reported
+                int64_t pos = valid ? (int64_t)p.rope_pos[row] : 0;
+                if (pos < 0 || pos >= p.max_pos) {
+                    set_status(p.status, KVB_ERR_INVALID_ARG);
+                    pos = 0;
+                }
+                const float* crow = p.cos_t + pos * (HD / 2);
+                const float* srow = p.sin_t + pos * (HD / 2);
                 const int64_t dst = valid ? (p.kv_dst ? (int64_t)p.kv_dst[row] : row) : 0;
+                const bool dst_ok = dst >= 0 && dst < p.n_kv_rows;
 #pragma unroll 1
                 for (int hh = 0; hh < NH; ++hh) {
                     const int c0 = tn * BN + hh * HD;          // column within this GEMM
                     if (c0 >= p.N) break;
                     const int colL = p.col_base + c0;          // column within [q | k | v]
                     uint16_t* outp;
-                    bool rope = true;
+                    uint16_t* outp2 = nullptr;   // bf16 copy of v (chunk-cache format)
+                    bool rope = true, write = valid;
                     if (colL < p.q_dim) {
                         outp = p.q_out + row * p.q_dim + colL;
                     } else if (colL < p.q_dim + p.kv_dim) {
                         outp = p.k_out + dst * p.kv_dim + (colL - p.q_dim);
+                        write = valid && dst_ok;
                     } else {
                         outp = p.v_out + dst * p.kv_dim + (colL - p.q_dim - p.kv_dim);
+                        if (p.v_out_bf16) outp2 = p.v_out_bf16 + dst * p.kv_dim + (colL - p.q_dim - p.kv_dim);
                         rope = false;
+                        write = valid && dst_ok;
                     }
+                    if (valid && !dst_ok && colL >= p.q_dim) set_status(p.status, KVB_ERR_INVALID_ARG);
                     const uint32_t tcol = taddr + (uint32_t)(hh * HD);
                     if (rope) {
 #pragma unroll 1
@@ -217,7 +230,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                             tmem_ld16(tcol + c * 16, x1);
                             tmem_ld16(tcol + HD / 2 + c * 16, x2);
                             tmem_ld_wait();
-                            if (valid) {
+                            if (write) {
                                 if (p.bias) {
                                     add_bias16(x1, p.bias + colL + c * 16);
                                     add_bias16(x2, p.bias + colL + HD / 2 + c * 16);
@@ -248,12 +261,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                             uint32_t x1[16];
                             tmem_ld16(tcol + c * 16, x1);
                             tmem_ld_wait();
-                            if (valid) {
+                            if (write) {
                                 if (p.bias) add_bias16(x1, p.bias + colL + c * 16);
                                 float y[16];
 #pragma unroll
                                 for (int i = 0; i < 16; ++i) y[i] = __uint_as_float(x1[i]);
                                 store16_bf16_as_f16(outp + c * 16, y);
+                                if (outp2) store16_bf16(outp2 + c * 16, y);
                             }
                         }
                     }

@@ -13,6 +13,13 @@ namespace kvb {
 
 // Record a message for kvb_last_error() and return the status.
 kvb_status fail(kvb_status s, const char* fmt, ...);
+// Clear the calling thread's kvb_last_error() message (every entry point does this first).
+void clear_last_error();
+// Argument checks shared by the entry points; each records a message when it fails.
+kvb_status check_cfg(const kvb_config* c);
+kvb_status check_ptr(const void* p, const char* name);
+kvb_status check_weights(const kvb_layer_weights* w);
+kvb_status check_rope(const kvb_rope_table* r, int64_t need_pos);
 // KVB_OK, or KVB_ERR_CUDA with the CUDA error text.
 kvb_status cuda_ok(cudaError_t e, const char* what);
 // Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current device the first time
@@ -47,7 +54,12 @@ struct GemmParams {
     uint16_t* k_out;
     uint16_t* v_out;
     const int32_t* kv_dst;
+    int64_t n_kv_rows;            // rows k_out / v_out hold: a row whose destination (kv_dst[r], or r)
+                                  // lies outside [0, n_kv_rows) writes no k / v and is reported
+    uint16_t* v_out_bf16;         // optional second copy of v in bf16 (the chunk-cache format), same rows
     const int32_t* rope_pos;
+    int64_t max_pos;              // rows of the RoPE tables: a position outside [0, max_pos) is reported
+                                  // and rotated by position 0
     const float* cos_t;
     const float* sin_t;
     const float* bias;            // fp32 bias of the [q | k | v] columns (added before RoPE), or NULL
@@ -81,10 +93,13 @@ kvb_status launch_attn(const AttnParams& p, const uint16_t* q, const uint16_t* k
 
 // ---------------------------------------------------------------- memory-bound kernels
 
+// K rotated by the chunk offset (bf16 -> bf16); V converted from the chunk caches' bf16 to the
+// blended cache's fp16 containers (a value outside fp16's finite range records KVB_ERR_RANGE
+// in *status and is written saturated to +-65504)
 kvb_status launch_realign(const float* cos_t, const float* sin_t, int D, int Hkv, const uint16_t* k_src,
                           const uint16_t* v_src, int64_t src_layer_stride, uint16_t* k_dst, uint16_t* v_dst,
                           int64_t dst_layer_stride, int n_layers, const int32_t* chunk_start, int n_chunks,
-                          int64_t n_ctx, cudaStream_t st);
+                          int64_t n_ctx, int* status, cudaStream_t st);
 // token ids outside [0, vocab) give a zero row and KVB_ERR_INVALID_ARG in *status
 kvb_status launch_embed(const uint16_t* embed, const int32_t* tok, int64_t n, int H, int vocab, float* x,
                         int* status, cudaStream_t st);

@@ -10,6 +10,9 @@
 // The array is sized for KVB_NOALLOC_MAX_ELEMS bf16 values (8 MiB); every GPU that
 // loads the library holds it until the process exits.  All calls share it: two calls
 // whose kernels overlap on the GPU (different streams without ordering) race on it.
+// Its device address is looked up once per device and kept for the life of the process,
+// so the entry point must not be used on a device after cudaDeviceReset() there (the
+// module is reloaded and the array may move).
 #include <mutex>
 
 #include "common.cuh"
@@ -55,28 +58,31 @@ extern "C" kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, cons
                                                      const kvb_rope_table* rope, const float* x,
                                                      const int32_t* row_idx, const int32_t* rope_pos, int64_t m,
                                                      uint16_t* q_out, uint16_t* k_out, uint16_t* v_out,
-                                                     const int32_t* kv_dst, int32_t* status_out, void* stream) {
-    if (!cfg || !w || !rope) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: config, weights or rope table is NULL");
-    if (m < 0) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: m < 0");
+                                                     const int32_t* kv_dst, int64_t n_kv_rows, int32_t* status_out,
+                                                     void* stream) {
+    // the same validation as kvb_gather_rmsnorm_qkv, so both entry points accept and reject the same inputs
+    clear_last_error();
+    kvb_status s = check_cfg(cfg);
+    if (s != KVB_OK) return s;
+    if ((s = check_weights(w)) != KVB_OK) return s;
+    if (m < 0 || n_kv_rows < 0) return fail(KVB_ERR_INVALID_ARG, "m < 0 or n_kv_rows < 0");
     if (m == 0) return KVB_OK;
-    if (cfg->hidden <= 0 || (size_t)m * (size_t)cfg->hidden > kNoAllocMaxElems)
+    const void* ptrs[] = {x, rope_pos, q_out, k_out, v_out};
+    const char* names[] = {"x", "rope_pos", "q_out", "k_out", "v_out"};
+    for (int i = 0; i < 5; ++i)
+        if ((s = check_ptr(ptrs[i], names[i])) != KVB_OK) return s;
+    if ((s = check_rope(rope, 1)) != KVB_OK) return s;
+    if (status_out && !aligned16(status_out))
+        return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: status_out not 16-byte aligned");
+    // the one limit of its own: the normalised rows must fit the fixed scratch
+    if ((size_t)m * (size_t)cfg->hidden > kNoAllocMaxElems)
         return fail(KVB_ERR_INVALID_ARG,
                     "no-alloc qkv: m * hidden = %lld exceeds the fixed scratch of %lld elements (use "
                     "kvb_gather_rmsnorm_qkv with a workspace, or split the rows)",
                     (long long)m * cfg->hidden, (long long)kNoAllocMaxElems);
-    if (cfg->head_dim != 64 && cfg->head_dim != 128)
-        return fail(KVB_ERR_UNSUPPORTED, "no-alloc qkv: head_dim %d not built", cfg->head_dim);
-    if (cfg->n_kv_heads <= 0 || cfg->n_q_heads % cfg->n_kv_heads || cfg->hidden % 256)
-        return fail(KVB_ERR_UNSUPPORTED, "no-alloc qkv: unsupported head counts or hidden size");
-    const void* ptrs[] = {w->attn_norm, w->w_qkv, x, rope_pos, q_out, k_out, v_out, rope->cos, rope->sin};
-    for (const void* p : ptrs)
-        if (!p || !aligned16(p)) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: NULL or misaligned pointer");
-    if (status_out && !aligned16(status_out))
-        return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: status_out not 16-byte aligned");
-    if (w->b_qkv && !aligned16(w->b_qkv)) return fail(KVB_ERR_INVALID_ARG, "no-alloc qkv: b_qkv not 16-byte aligned");
 
     void* scratch = nullptr;
-    kvb_status s = scratch_address(&scratch);
+    s = scratch_address(&scratch);
     if (s != KVB_OK) return s;
     uint16_t* a = static_cast<uint16_t*>(scratch);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -88,7 +94,8 @@ extern "C" kvb_status kvb_gather_rmsnorm_qkv_noalloc(const kvb_config* cfg, cons
     GemmParams p{};
     p.M = m; p.N = QD + 2 * KVD; p.K = H; p.epi = EPI_QKV;
     p.col_base = 0; p.q_dim = QD; p.kv_dim = KVD; p.head_dim = D;
-    p.q_out = q_out; p.k_out = k_out; p.v_out = v_out; p.kv_dst = kv_dst; p.rope_pos = rope_pos;
+    p.q_out = q_out; p.k_out = k_out; p.v_out = v_out; p.kv_dst = kv_dst; p.n_kv_rows = n_kv_rows;
+    p.rope_pos = rope_pos; p.max_pos = rope->max_pos;
     p.cos_t = rope->cos; p.sin_t = rope->sin; p.bias = w->b_qkv; p.status = status_out;
     return launch_gemm(p, a, H, w->w_qkv, H, nullptr, st);
 }

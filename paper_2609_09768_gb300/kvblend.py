@@ -28,8 +28,9 @@ class KvbError(RuntimeError):
 
 
 STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "CUDA error", 4: "device wait timed out",
-          5: "workspace too small"}
-KVB_OK, KVB_ERR_INVALID_ARG, KVB_ERR_UNSUPPORTED, KVB_ERR_CUDA, KVB_ERR_TIMEOUT, KVB_ERR_WORKSPACE = range(6)
+          5: "workspace too small", 6: "value out of range"}
+(KVB_OK, KVB_ERR_INVALID_ARG, KVB_ERR_UNSUPPORTED, KVB_ERR_CUDA, KVB_ERR_TIMEOUT, KVB_ERR_WORKSPACE,
+ KVB_ERR_RANGE) = range(7)
 KVB_ROPE_PLAIN, KVB_ROPE_LLAMA3, KVB_ROPE_YARN = range(3)
 
 
@@ -67,6 +68,11 @@ class Timings(C.Structure):
         return {f: getattr(self, f) for f, _ in self._fields_}
 
 
+class LayerTapsStruct(C.Structure):
+    _fields_ = [("n", c_i32), ("layers", C.POINTER(c_i32)), ("x_out", c_vp), ("rows_cap", c_i64),
+                ("rows_out", C.POINTER(c_i64))]
+
+
 P = C.POINTER
 _SIGS = {
     "kvb_status_string": (C.c_char_p, [c_i32]),
@@ -75,13 +81,13 @@ _SIGS = {
     "kvb_rope_table_fill": (c_i32, [P(Config), c_i64, c_vp, c_vp]),
     "kvb_attention_scale": (c_i32, [P(Config), P(c_f32)]),
     "kvb_rope_realign": (c_i32, [P(Config), P(RopeTableStruct), c_vp, c_vp, c_i64, c_vp, c_vp, c_i64, c_i32, c_i32,
-                                 c_vp, c_i32, c_i64, c_vp]),
+                                 c_vp, c_i32, c_i64, c_vp, c_sz, c_vp]),
     "kvb_hkvd_workspace_size": (c_sz, [c_i64]),
     "kvb_hkvd_select": (c_i32, [c_vp, c_i64, c_vp, c_i64, c_i64, c_i32, c_i64, c_vp, c_vp, c_vp, c_sz, c_vp]),
     "kvb_gather_rmsnorm_qkv": (c_i32, [P(Config), P(LayerWeights), P(RopeTableStruct), c_vp, c_vp, c_vp, c_i64,
-                                       c_vp, c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]),
+                                       c_vp, c_vp, c_vp, c_vp, c_i64, c_vp, c_sz, c_vp]),
     "kvb_gather_rmsnorm_qkv_noalloc": (c_i32, [P(Config), P(LayerWeights), P(RopeTableStruct), c_vp, c_vp, c_vp,
-                                               c_i64, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
+                                               c_i64, c_vp, c_vp, c_vp, c_vp, c_i64, c_vp, c_vp]),
     "kvb_kv_scatter": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i32, c_vp, c_vp, c_i64, c_vp]),
     "kvb_sparse_query_attn": (c_i32, [P(Config), c_vp, c_vp, c_vp, c_i64, c_vp, c_vp, c_i64, c_vp, c_vp, c_sz,
                                       c_vp]),
@@ -89,13 +95,13 @@ _SIGS = {
     "kvb_workspace_size": (c_i32, [P(Config), c_i64, P(c_sz)]),
     "kvb_selective_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), c_vp, c_vp, P(KVCache), c_vp,
                                       c_vp, c_i32, c_i64, c_i64, c_f32, c_i32, c_vp, c_i64, c_vp, c_vp, P(Timings),
-                                      c_vp, c_sz, c_vp]),
+                                      P(LayerTapsStruct), c_vp, c_sz, c_vp]),
     "kvb_selective_prefill_host": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), c_vp, c_vp, P(KVCache),
                                            c_vp, c_vp, c_i32, c_i64, c_i64, c_f32, c_i32, c_vp, c_i64, c_vp, c_vp,
-                                           P(Timings), c_vp, c_sz, c_vp, c_vp]),
+                                           P(Timings), P(LayerTapsStruct), c_vp, c_sz, c_vp, c_vp]),
     "kvb_workspace_size_pipelined": (c_i32, [P(Config), c_i64, c_i64, P(c_sz)]),
-    "kvb_full_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), P(KVCache), c_vp, c_i64, c_vp, c_vp,
-                                 c_vp, c_i64, P(Timings), c_vp, c_sz, c_vp]),
+    "kvb_full_prefill": (c_i32, [P(Config), P(ModelStruct), P(RopeTableStruct), P(KVCache), c_vp, c_vp, c_i64, c_vp,
+                                 c_vp, c_vp, c_i64, P(Timings), P(LayerTapsStruct), c_vp, c_sz, c_vp]),
     "kvb_device_status": (c_i32, [c_vp, c_sz, c_vp, P(c_i32)]),
     "kvb_debug_wait_timeout": (c_i32, [c_vp, c_sz, c_i64, c_vp]),
     "kvb_lm_head_argmax": (c_i32, [P(Config), c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_sz, c_vp]),
@@ -208,9 +214,34 @@ class Model:
 
 
 def kv_cache_struct(k: torch.Tensor, v: torch.Tensor) -> KVCache:
-    """k: [L][n_rows][Hkv][D] bf16; v: same shape, fp16 (bf16-precision values)."""
+    """Blended cache: k [L][n_rows][Hkv][D] bf16; v the same shape, fp16 (bf16-precision values)."""
     assert k.shape == v.shape and k.dim() == 4
     return KVCache(_ptr(k, torch.bfloat16, "cache k"), _ptr(v, torch.float16, "cache v"), k.shape[1], k.shape[0])
+
+
+class LayerTaps:
+    """Residual rows captured at layer boundaries (kvb_layer_taps): slot i holds the fp32 rows
+    entering layer layers[i] (n_layers: leaving the last layer), rows_cap rows per slot.
+    After the call, `rows(i)` is the number of rows captured in slot i and `get(i)` the
+    [rows][H] view of them."""
+
+    def __init__(self, layers, rows_cap: int, hidden: int, device="cuda"):
+        self.layers = list(int(l) for l in layers)
+        self.hidden = hidden
+        self.x = torch.zeros(max(len(self.layers), 1), rows_cap, hidden, dtype=torch.float32, device=device)
+        self._layers = (c_i32 * max(len(self.layers), 1))(*self.layers)
+        self._rows = (c_i64 * max(len(self.layers), 1))()
+        self.struct = LayerTapsStruct(len(self.layers), self._layers, self.x.data_ptr(), rows_cap, self._rows)
+
+    def rows(self, i: int) -> int:
+        return int(self._rows[i])
+
+    def get(self, i: int) -> torch.Tensor:
+        return self.x[i, : self.rows(i)]
+
+
+def _taps(taps: Optional[LayerTaps]):
+    return C.byref(taps.struct) if taps is not None else None
 
 
 # ---------------------------------------------------------------------------------- workspace
@@ -300,11 +331,22 @@ def device_status(ws: torch.Tensor) -> int:
 # ---------------------------------------------------------------------------------- steps
 
 def rope_realign(cfg: Config, rope: RopeTable, k_src, v_src, k_dst, v_dst, layer_begin: int, layer_end: int,
-                 chunk_start: torch.Tensor, n_ctx: int) -> None:
+                 chunk_start: torch.Tensor, n_ctx: int, ws: Optional[torch.Tensor] = None) -> None:
+    """Chunk caches (k_src, v_src: bf16 [L][src_rows][Hkv][D]) -> blended-cache layers (k_dst bf16,
+    v_dst fp16).  v_src / v_dst may be None (V untouched); a V value outside fp16's range is
+    recorded as KVB_ERR_RANGE in the status word of `ws` (256 bytes, allocated if None)."""
+    if ws is None and v_src is not None and v_dst is not None:
+        ws = torch.zeros(256, dtype=torch.uint8, device=k_src.device)
+    if v_src is not None and v_dst is not None and v_src.data_ptr() == v_dst.data_ptr():
+        # in place: the same memory holds bf16 before and fp16 after the call
+        vs, vd = _ptr(v_src, None, "v_src"), _ptr(v_dst, None, "v_dst")
+    else:
+        vs, vd = _ptr(v_src, torch.bfloat16, "v_src"), _ptr(v_dst, torch.float16, "v_dst")
     _call("kvb_rope_realign", C.byref(cfg), C.byref(rope.struct), _ptr(k_src, torch.bfloat16, "k_src"),
-          _ptr(v_src, torch.float16, "v_src"), k_src.shape[1], _ptr(k_dst, torch.bfloat16, "k_dst"),
-          _ptr(v_dst, torch.float16, "v_dst"), k_dst.shape[1], layer_begin, layer_end,
-          _ptr(chunk_start, torch.int32, "chunk_start"), chunk_start.numel() - 1, n_ctx, _stream())
+          vs, k_src.shape[1], _ptr(k_dst, torch.bfloat16, "k_dst"),
+          vd, k_dst.shape[1], layer_begin, layer_end,
+          _ptr(chunk_start, torch.int32, "chunk_start"), chunk_start.numel() - 1, n_ctx,
+          _ptr(ws) if ws is not None else None, ws.numel() if ws is not None else 0, _stream())
 
 
 def hkvd_select(k_fresh: torch.Tensor, k_cached: torch.Tensor, k: int, sel_out=None, dev_out=None,
@@ -324,24 +366,30 @@ def hkvd_select(k_fresh: torch.Tensor, k_cached: torch.Tensor, k: int, sel_out=N
 
 
 def gather_rmsnorm_qkv(cfg: Config, lw: LayerWeights, rope: RopeTable, x: torch.Tensor, row_idx, rope_pos, m: int,
-                       q_out, k_out, v_out, kv_dst, ws: torch.Tensor) -> None:
+                       q_out, k_out, v_out, kv_dst, ws: torch.Tensor, n_kv_rows: Optional[int] = None) -> None:
+    """k_out / v_out hold n_kv_rows rows (default: k_out's first dimension)."""
+    if n_kv_rows is None:
+        n_kv_rows = k_out.shape[0]
     _call("kvb_gather_rmsnorm_qkv", C.byref(cfg), C.byref(lw), C.byref(rope.struct), _ptr(x, torch.float32, "x"),
           _ptr(row_idx, torch.int32, "row_idx"), _ptr(rope_pos, torch.int32, "rope_pos"), m,
           _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"), _ptr(v_out, torch.float16, "v_out"),
-          _ptr(kv_dst, torch.int32, "kv_dst"), _ptr(ws), ws.numel(), _stream())
+          _ptr(kv_dst, torch.int32, "kv_dst"), n_kv_rows, _ptr(ws), ws.numel(), _stream())
 
 
 NOALLOC_MAX_ELEMS = 4 * 1024 * 1024
 
 
 def gather_rmsnorm_qkv_noalloc(cfg: Config, lw: LayerWeights, rope: RopeTable, x: torch.Tensor, row_idx, rope_pos,
-                               m: int, q_out, k_out, v_out, kv_dst, status_out: Optional[torch.Tensor] = None) -> None:
+                               m: int, q_out, k_out, v_out, kv_dst, status_out: Optional[torch.Tensor] = None,
+                               n_kv_rows: Optional[int] = None) -> None:
     """kvb_gather_rmsnorm_qkv without a workspace: the library's fixed scratch holds the
     normalised rows (m * hidden <= NOALLOC_MAX_ELEMS), for callers that cannot allocate."""
+    if n_kv_rows is None:
+        n_kv_rows = k_out.shape[0]
     _call("kvb_gather_rmsnorm_qkv_noalloc", C.byref(cfg), C.byref(lw), C.byref(rope.struct),
           _ptr(x, torch.float32, "x"), _ptr(row_idx, torch.int32, "row_idx"), _ptr(rope_pos, torch.int32, "rope_pos"),
           m, _ptr(q_out, torch.bfloat16, "q_out"), _ptr(k_out, torch.bfloat16, "k_out"),
-          _ptr(v_out, torch.float16, "v_out"), _ptr(kv_dst, torch.int32, "kv_dst"),
+          _ptr(v_out, torch.float16, "v_out"), _ptr(kv_dst, torch.int32, "kv_dst"), n_kv_rows,
           _ptr(status_out, torch.int32, "status_out"), _stream())
 
 
@@ -370,8 +418,10 @@ def mlp_rows(cfg: Config, lw: LayerWeights, attn, x, ws: torch.Tensor) -> None:
 def selective_prefill(cfg: Config, model: Model, rope: RopeTable, k_chunks, v_chunks, cache_k, cache_v, token_ids,
                       chunk_start: torch.Tensor, n_ctx: int, n_query: int, r: float, check_layer: int = 1,
                       forced_sel: Optional[torch.Tensor] = None, final_hidden=None, sel_out=None,
-                      ws: Optional[torch.Tensor] = None, timings: bool = False):
-    """Runs kvb_selective_prefill.  Returns (final_hidden [n_query][H] fp32, sel_out, timings dict or None)."""
+                      ws: Optional[torch.Tensor] = None, timings: bool = False, taps: Optional[LayerTaps] = None):
+    """Runs kvb_selective_prefill on chunk caches k_chunks / v_chunks (bf16 [L][n_ctx][Hkv][D]) into the
+    blended cache (cache_k bf16, cache_v fp16).  Returns (final_hidden [n_query][H] fp32, sel_out,
+    timings dict or None)."""
     dev = token_ids.device
     if final_hidden is None:
         final_hidden = torch.empty(max(n_query, 1), cfg.hidden, dtype=torch.float32, device=dev)
@@ -382,12 +432,12 @@ def selective_prefill(cfg: Config, model: Model, rope: RopeTable, k_chunks, v_ch
     cache = kv_cache_struct(cache_k, cache_v)
     t = Timings()
     _call("kvb_selective_prefill", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct),
-          _ptr(k_chunks, torch.bfloat16, "k_chunks"), _ptr(v_chunks, torch.float16, "v_chunks"), C.byref(cache),
+          _ptr(k_chunks, torch.bfloat16, "k_chunks"), _ptr(v_chunks, torch.bfloat16, "v_chunks"), C.byref(cache),
           _ptr(token_ids, torch.int32, "token_ids"), _ptr(chunk_start, torch.int32, "chunk_start"),
           (chunk_start.numel() - 1) if chunk_start is not None else 0, n_ctx, n_query, r, check_layer,
           _ptr(forced_sel, torch.int32, "forced_sel"), forced_sel.numel() if forced_sel is not None else 0,
           _ptr(final_hidden, torch.float32, "final_hidden"), _ptr(sel_out, torch.int32, "sel_out"),
-          C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream())
+          C.byref(t) if timings else None, _taps(taps), _ptr(ws), ws.numel(), _stream())
     return final_hidden[:n_query], sel_out, (t.as_dict() if timings else None)
 
 
@@ -409,7 +459,8 @@ def selective_prefill_host(cfg: Config, model: Model, rope: RopeTable, k_chunks_
                            token_ids, chunk_start: torch.Tensor, n_ctx: int, n_query: int, r: float,
                            check_layer: int = 1, copy_stream: Optional[torch.cuda.Stream] = None,
                            forced_sel: Optional[torch.Tensor] = None, final_hidden=None, sel_out=None,
-                           ws: Optional[torch.Tensor] = None, timings: bool = False):
+                           ws: Optional[torch.Tensor] = None, timings: bool = False,
+                           taps: Optional[LayerTaps] = None):
     """kvb_selective_prefill_host: chunk caches in pinned host memory, ingested layer by layer
     on `copy_stream` under the compute on the current stream."""
     dev = token_ids.device
@@ -424,18 +475,21 @@ def selective_prefill_host(cfg: Config, model: Model, rope: RopeTable, k_chunks_
     cache = kv_cache_struct(cache_k, cache_v)
     t = Timings()
     _call("kvb_selective_prefill_host", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct),
-          _host_ptr(k_chunks_host, torch.bfloat16, "k_chunks_host"), _host_ptr(v_chunks_host, torch.float16, "v_chunks_host"),
+          _host_ptr(k_chunks_host, torch.bfloat16, "k_chunks_host"), _host_ptr(v_chunks_host, torch.bfloat16, "v_chunks_host"),
           C.byref(cache), _ptr(token_ids, torch.int32, "token_ids"), _ptr(chunk_start, torch.int32, "chunk_start"),
           chunk_start.numel() - 1, n_ctx, n_query, r, check_layer,
           _ptr(forced_sel, torch.int32, "forced_sel"), forced_sel.numel() if forced_sel is not None else 0,
           _ptr(final_hidden, torch.float32, "final_hidden"), _ptr(sel_out, torch.int32, "sel_out"),
-          C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream(), copy_stream.cuda_stream)
+          C.byref(t) if timings else None, _taps(taps), _ptr(ws), ws.numel(), _stream(), copy_stream.cuda_stream)
     return final_hidden[:n_query], sel_out, (t.as_dict() if timings else None)
 
 
 def full_prefill(cfg: Config, model: Model, rope: RopeTable, cache_k, cache_v, token_ids, rope_pos=None, kv_lo=None,
-                 n_out: int = 0, final_hidden=None, ws: Optional[torch.Tensor] = None, timings: bool = False):
-    """Runs kvb_full_prefill over all rows of token_ids.  Returns (final_hidden or None, timings or None)."""
+                 n_out: int = 0, final_hidden=None, ws: Optional[torch.Tensor] = None, timings: bool = False,
+                 v_chunk_out: Optional[torch.Tensor] = None, taps: Optional[LayerTaps] = None):
+    """Runs kvb_full_prefill over all rows of token_ids into the blended cache (cache_k bf16, cache_v
+    fp16); v_chunk_out (bf16 [L][n][Hkv][D]) also receives every layer's V in the chunk-cache format.
+    Returns (final_hidden or None, timings or None)."""
     n = token_ids.numel()
     dev = token_ids.device
     if n_out and final_hidden is None:
@@ -445,9 +499,10 @@ def full_prefill(cfg: Config, model: Model, rope: RopeTable, cache_k, cache_v, t
     cache = kv_cache_struct(cache_k, cache_v)
     t = Timings()
     _call("kvb_full_prefill", C.byref(cfg), C.byref(model.struct), C.byref(rope.struct), C.byref(cache),
+          _ptr(v_chunk_out, torch.bfloat16, "v_chunk_out"),
           _ptr(token_ids, torch.int32, "token_ids"), n, _ptr(rope_pos, torch.int32, "rope_pos"),
           _ptr(kv_lo, torch.int32, "kv_lo"), _ptr(final_hidden, torch.float32, "final_hidden") if n_out else None,
-          n_out, C.byref(t) if timings else None, _ptr(ws), ws.numel(), _stream())
+          n_out, C.byref(t) if timings else None, _taps(taps), _ptr(ws), ws.numel(), _stream())
     return final_hidden, (t.as_dict() if timings else None)
 
 

@@ -33,15 +33,17 @@ def chunk_layout(chunk_starts: List[int], device="cuda"):
 
 def chunk_caches(cfg: kvb.Config, model: kvb.Model, rope: kvb.RopeTable, ctx_tokens: torch.Tensor,
                  chunk_starts: List[int], ws: Optional[torch.Tensor] = None, zero_rows: Optional[List[int]] = None):
-    """Per-chunk caches [L][n_ctx][Hkv][D] (keys at chunk-local positions; K bf16, V fp16).
-    Rows in `zero_rows` (separator tokens) are set to zero in every layer."""
+    """Per-chunk caches in the chunk-cache format: K and V bf16 [L][n_ctx][Hkv][D], keys at
+    chunk-local positions.  Rows in `zero_rows` (separator tokens) are set to zero in every layer."""
     n_ctx = chunk_starts[-1]
     L = cfg.n_layers
     dev = ctx_tokens.device
     k = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.bfloat16, device=dev)
-    v = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.float16, device=dev)
+    v = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.bfloat16, device=dev)
+    v_att = torch.empty(L, n_ctx, cfg.n_kv_heads, cfg.head_dim, dtype=torch.float16, device=dev)  # read by attention
     pos, lo = chunk_layout(chunk_starts, dev)
-    kvb.full_prefill(cfg, model, rope, k, v, ctx_tokens, rope_pos=pos, kv_lo=lo, ws=ws)
+    kvb.full_prefill(cfg, model, rope, k, v_att, ctx_tokens, rope_pos=pos, kv_lo=lo, ws=ws, v_chunk_out=v)
+    del v_att
     if zero_rows:
         idx = torch.tensor(zero_rows, dtype=torch.long, device=dev)
         k[:, idx] = 0

@@ -100,7 +100,7 @@ def test_host_validation_rejects_bad_arguments(kvb):
     # NULL config / pointers are rejected before any device work
     assert L.kvb_rope_table_fill(None, 10, None, None) == kvb.KVB_ERR_INVALID_ARG
     assert L.kvb_selective_prefill(None, None, None, None, None, None, None, None, 0, 0, 0, 0.15, 1, None, 0, None,
-                                   None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+                                   None, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
     assert b"config is NULL" in L.kvb_last_error()
     bad = kvb.config(synth.TINY)
     bad.head_dim = 96
@@ -118,7 +118,7 @@ def test_host_validation_rejects_bad_arguments(kvb):
     # r outside [0, 1] and a check layer outside [1, L]
     mw = kvb.ModelStruct()
     assert L.kvb_selective_prefill(C.byref(cfg), C.byref(mw), None, None, None, None, None, None, 1, 10, 2, 1.5, 1,
-                                   None, 0, None, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
+                                   None, 0, None, None, None, None, None, 0, None) == kvb.KVB_ERR_INVALID_ARG
     assert L.kvb_debug_wait_timeout(None, 0, 10**6, None) == kvb.KVB_ERR_INVALID_ARG
     # empty inputs are valid no-ops
     assert L.kvb_kv_scatter(None, None, None, 0, 128, None, None, 4, None) == kvb.KVB_OK
@@ -153,3 +153,71 @@ def test_shape_from_published_config_layout():
     assert plain.rope_scaling == 0 and plain.head_dim == 64
     with pytest.raises(ValueError):
         synth.shape_from_config(dict(base, rope_scaling={"type": "dynamic", "factor": 2.0}))
+
+
+def test_both_qkv_entry_points_validate_alike(kvb):
+    """The workspace and the allocation-free QKV entry points accept and reject the same
+    configurations (they share one validation); a failed call leaves a message, and the next
+    successful validation step clears it."""
+    L = kvb.lib()
+    lw = kvb.LayerWeights(16, 16, 16, 16, 16, 16, 16, None)
+    for hq, hkv in ((0, 2), (-2, 2), (4, 0)):
+        bad = kvb.config(synth.TINY)
+        bad.n_q_heads, bad.n_kv_heads = hq, hkv
+        a = L.kvb_gather_rmsnorm_qkv(C.byref(bad), C.byref(lw), None, None, None, None, 4, None, None, None, None,
+                                     8, None, 0, None)
+        msg_a = L.kvb_last_error()
+        b = L.kvb_gather_rmsnorm_qkv_noalloc(C.byref(bad), C.byref(lw), None, None, None, None, 4, None, None, None,
+                                             None, 8, None, None)
+        msg_b = L.kvb_last_error()
+        assert a == b == kvb.KVB_ERR_INVALID_ARG, (hq, hkv, a, b)
+        assert msg_a == msg_b and msg_a
+    good = kvb.config(synth.TINY)
+    # a bad eps / theta and an unknown scaling are rejected by both as well
+    for field, value in (("rms_eps", -1.0), ("rope_theta", 0.0), ("rope_scaling", 9)):
+        bad = kvb.config(synth.TINY)
+        setattr(bad, field, value)
+        a = L.kvb_gather_rmsnorm_qkv(C.byref(bad), C.byref(lw), None, None, None, None, 4, None, None, None, None,
+                                     8, None, 0, None)
+        b = L.kvb_gather_rmsnorm_qkv_noalloc(C.byref(bad), C.byref(lw), None, None, None, None, 4, None, None, None,
+                                             None, 8, None, None)
+        assert a == b == kvb.KVB_ERR_INVALID_ARG, field
+    # with a valid config, m == 0 is a no-op for both and clears the previous message
+    assert L.kvb_gather_rmsnorm_qkv(C.byref(good), C.byref(lw), None, None, None, None, 0, None, None, None, None, 0,
+                                    None, 0, None) == kvb.KVB_OK
+    assert L.kvb_last_error() == b""
+    assert L.kvb_gather_rmsnorm_qkv_noalloc(C.byref(good), C.byref(lw), None, None, None, None, 0, None, None, None,
+                                            None, 0, None, None) == kvb.KVB_OK
+    assert L.kvb_last_error() == b""
+    # a NULL rope table is rejected by both once there are rows to compute
+    assert L.kvb_gather_rmsnorm_qkv(C.byref(good), C.byref(lw), None, 16, None, 16, 4, 16, 16, 16, None, 8, None, 0,
+                                    None) == kvb.KVB_ERR_INVALID_ARG
+    assert L.kvb_gather_rmsnorm_qkv_noalloc(C.byref(good), C.byref(lw), None, 16, None, 16, 4, 16, 16, 16, None, 8,
+                                            None, None) == kvb.KVB_ERR_INVALID_ARG
+
+
+def test_layer_taps_are_validated_before_any_launch(kvb):
+    """A tap outside [0, n_layers] or one that needs more rows than its slots hold fails the
+    call with INVALID_ARG before anything runs.  The device pointers here are stand-ins that
+    validation only checks for alignment; no GPU is needed because nothing is launched."""
+    L = kvb.lib()
+    cfg = kvb.config(synth.TINY)                       # 2 layers
+    fake = 1 << 20                                     # aligned, never dereferenced
+    lws = (kvb.LayerWeights * cfg.n_layers)(*[kvb.LayerWeights(fake, fake, fake, fake, fake, fake, fake, None)
+                                               for _ in range(cfg.n_layers)])
+    mw = kvb.ModelStruct(C.cast(lws, C.POINTER(kvb.LayerWeights)), fake, fake)
+    rope = kvb.RopeTableStruct(fake, fake, 1000)
+    n = 300
+    cache = kvb.KVCache(fake, fake, n, cfg.n_layers)
+
+    def call(layer, rows_cap):
+        layers = (C.c_int32 * 1)(layer)
+        taps = kvb.LayerTapsStruct(1, layers, fake, rows_cap, None)
+        return L.kvb_full_prefill(C.byref(cfg), C.byref(mw), C.byref(rope), C.byref(cache), None, fake, n, None,
+                                  None, None, 0, None, C.byref(taps), None, 0, None)
+
+    assert call(3, n) == kvb.KVB_ERR_INVALID_ARG and b"taps: layer 3 not in [0, 2]" in L.kvb_last_error()
+    assert call(-1, n) == kvb.KVB_ERR_INVALID_ARG
+    assert call(1, n - 1) == kvb.KVB_ERR_INVALID_ARG and b"carries 300 rows" in L.kvb_last_error()
+    # a valid tap passes validation and the call stops at the (missing) workspace instead
+    assert call(2, n) == kvb.KVB_ERR_WORKSPACE

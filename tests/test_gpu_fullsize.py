@@ -9,7 +9,8 @@ import torch
 from oracle import blend, llama
 from oracle.llama import Shape
 from paper_2609_09768_gb300 import synth, workload
-from tests.gpu_util import assert_close_abs, assert_close_bf16, assert_close_rel, np64
+from tests.attn_cases import TILE, assert_attn_close, peaked_queries, tagged_case
+from tests.gpu_util import assert_close_abs, assert_close_bf16, np64
 
 pytestmark = pytest.mark.gpu
 
@@ -38,31 +39,75 @@ def sample_rows(m, k=48, seed=0):
     return s
 
 
-@pytest.mark.parametrize("mode", ["selective", "dense"])
-def test_attention_full_size_sampled_rows(kvb, mode):
-    cfg = kvb.config(SHAPE)
-    g = gen(1)
+def residue_sample(hi, lo, k=256, seed=0):
+    """Indices of k rows: for every residue of a 144-key tile, a row whose own key hi (and,
+    where ranges start inside the cache, a row whose first key lo) sits on it, then the first,
+    middle and last rows, the rest uniform."""
+    hi, lo = np.asarray(hi), np.asarray(lo)
+    pick = set()
+    for res in range(TILE):
+        for arr in ((hi,) if not lo.any() else (hi, lo)):
+            idx = np.nonzero(arr % TILE == res)[0]
+            if len(idx):
+                pick.add(int(idx[len(idx) // 2]))
+    m = len(hi)
+    pick.update([0, 1, m // 2, m - 2, m - 1])
+    rng = np.random.default_rng(seed)
+    rest = np.setdiff1d(np.arange(m), sorted(pick))
+    if len(pick) < k:
+        pick.update(rng.choice(rest, k - len(pick), replace=False).tolist())
+    return np.array(sorted(pick))
+
+
+def _full_size_rows(mode, g):
     if mode == "dense":
         rows = torch.arange(N, dtype=torch.int32, device="cuda")
+        lo = None
+    elif mode == "block_diagonal":            # the per-chunk prefill that builds the chunk caches
+        rows = torch.arange(N_CTX, dtype=torch.int32, device="cuda")
+        lo = torch.div(rows, WL.chunk_len, rounding_mode="floor").to(torch.int32) * WL.chunk_len
     else:
         perm = torch.randperm(N_CTX, generator=g, device="cuda")[: M_SEL - WL.n_query]
-        rows = torch.cat([torch.sort(perm).values,
-                          torch.arange(N_CTX, N, device="cuda")]).to(torch.int32)
+        rows = torch.cat([torch.sort(perm).values, torch.arange(N_CTX, N, device="cuda")]).to(torch.int32)
+        lo = None
+    return rows, lo
+
+
+@pytest.mark.parametrize("tagged", [False, True])
+@pytest.mark.parametrize("mode", ["selective", "dense", "block_diagonal"])
+def test_attention_full_size_sampled_rows(kvb, mode, tagged):
+    """The attention launches of the headline request at full size (18,713 selected rows
+    or all 124,032 rows over the 124,032-row cache; the 123,904-row block-diagonal prefill of
+    the 512-token chunks), judged on >= 256 sampled rows, all heads, that put a row's own
+    key (and first key) on every residue of a 144-key tile.  Inputs: peaked random queries,
+    or tagged keys (each (row, head) reads one chosen key: its own, the next one, the first
+    or the one before its range, a tile edge, ...)."""
+    cfg = kvb.config(SHAPE)
+    g = gen(1)
+    rows, lo = _full_size_rows(mode, g)
     m = rows.numel()
-    q = torch.randn(m, SHAPE.n_q_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
-    k = torch.randn(N, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
-    v = torch.randn(N, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16).to(torch.float16)
+    n_kv = N_CTX if mode == "block_diagonal" else N
+    hi_np = rows.cpu().numpy().astype(np.int64)
+    lo_np = lo.cpu().numpy().astype(np.int64) if lo is not None else np.zeros(m, dtype=np.int64)
+    if tagged:
+        q, k, v, _ = tagged_case(n_kv, hi_np, lo_np, SHAPE.n_q_heads, SHAPE.n_kv_heads, SHAPE.head_dim, seed=5)
+        q, k, v = q.cuda(), k.cuda(), v.to(torch.float16).cuda()
+    else:
+        q = peaked_queries(m, SHAPE.n_q_heads, SHAPE.head_dim, seed=5).cuda()
+        k = torch.randn(n_kv, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
+        v = torch.randn(n_kv, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(
+            torch.bfloat16).to(torch.float16)
     out = torch.empty(m, SHAPE.q_dim, dtype=torch.bfloat16, device="cuda")
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
-    kvb.sparse_query_attn(cfg, q, rows, None, k, v, out, ws)
+    kvb.sparse_query_attn(cfg, q, rows, lo, k, v, out, ws)
     torch.cuda.synchronize()
     assert kvb.device_status(ws) == 0
-    smp = sample_rows(m)
-    ri = rows.cpu().numpy()
-    ref = llama.attention_rows(Shape.of(SHAPE), np64(q.cpu()[smp]), np64(k.cpu()), np64(v.cpu()), ri[smp])
-    vs = float(np.sqrt(np.mean(np64(v.cpu()) ** 2)))
-    e = assert_close_rel(out.cpu()[smp], ref.reshape(len(smp), -1), f"{mode} attention at full size", scale=vs)
-    print(mode, m, e)
+    smp = residue_sample(hi_np, lo_np)
+    assert len(smp) >= 256
+    ref = llama.attention_rows(Shape.of(SHAPE), np64(q.cpu()[smp]), np64(k.cpu()), np64(v.cpu()), hi_np[smp],
+                               lo_np[smp] if lo is not None else None)
+    e = assert_attn_close(out.cpu()[smp], ref.reshape(len(smp), -1), f"{mode} attention at full size")
+    print(mode, "tagged" if tagged else "peaked", m, e)
 
 
 @pytest.mark.parametrize("m", [M_SEL, N])
@@ -104,14 +149,17 @@ def test_realign_full_size_sampled_rows(kvb):
     L = SHAPE.n_layers - 1
     g = gen(3)
     ks = torch.randn(L, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
-    vs = torch.randn(L, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.float16)
+    vs = torch.randn(L, N_CTX, SHAPE.n_kv_heads, SHAPE.head_dim, generator=g, device="cuda").to(torch.bfloat16)
     kd = torch.empty(L, N, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.bfloat16, device="cuda")
     vd = torch.empty(L, N, SHAPE.n_kv_heads, SHAPE.head_dim, dtype=torch.float16, device="cuda")
     rope = kvb.RopeTable(cfg, N)
     starts = WL.chunk_starts()
-    kvb.rope_realign(cfg, rope, ks, vs, kd, vd, 0, L, torch.tensor(starts, dtype=torch.int32, device="cuda"), N_CTX)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    kvb.rope_realign(cfg, rope, ks, vs, kd, vd, 0, L, torch.tensor(starts, dtype=torch.int32, device="cuda"), N_CTX,
+                     ws=ws)
     torch.cuda.synchronize()
-    assert torch.equal(vd[:, :N_CTX], vs)
+    assert kvb.device_status(ws) == kvb.KVB_OK
+    assert torch.equal(vd[:, :N_CTX], vs.to(torch.float16))
     smp = np.unique(np.concatenate([[0, 511, 512, N_CTX - 1], np.random.default_rng(4).choice(N_CTX, 60)]))
     got = kd[:, smp].cpu()
     # the oracle rotates each sampled row by its own chunk's offset

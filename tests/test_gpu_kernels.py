@@ -7,7 +7,8 @@ import torch
 from oracle import blend, llama
 from oracle.llama import Shape
 from paper_2609_09768_gb300 import synth
-from tests.gpu_util import (assert_close_abs, assert_close_bf16, assert_close_rel, check_selection, errs, np64)
+from tests.attn_cases import assert_attn_close, peaked_queries, tagged_case
+from tests.gpu_util import assert_close_abs, assert_close_bf16, check_selection, errs, np64
 
 pytestmark = pytest.mark.gpu
 
@@ -39,17 +40,26 @@ def test_realign_matches_oracle(kvb, shape, starts):
     cfg = kvb.config(shape)
     n_ctx, L, Hkv, D = starts[-1], shape.n_layers, shape.n_kv_heads, shape.head_dim
     k_src = synth.randn_bf16((L, n_ctx, Hkv, D), 101)
-    v_src = synth.randn_bf16((L, n_ctx, Hkv, D), 102).to(torch.float16)
+    v_src = synth.randn_bf16((L, n_ctx, Hkv, D), 102)            # chunk caches hold bf16 V
     rope = kvb.RopeTable(cfg, n_ctx)
     cs = dev(torch.tensor(starts, dtype=torch.int32))
     rows = n_ctx + 13
     k_dst = torch.zeros(L, rows, Hkv, D, dtype=torch.bfloat16, device="cuda")
     v_dst = torch.zeros(L, rows, Hkv, D, dtype=torch.float16, device="cuda")
-    kvb.rope_realign(cfg, rope, dev(k_src), dev(v_src), k_dst, v_dst, 0, L, cs, n_ctx)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    kvb.rope_realign(cfg, rope, dev(k_src), dev(v_src), k_dst, v_dst, 0, L, cs, n_ctx, ws=ws)
     torch.cuda.synchronize()
+    assert kvb.device_status(ws) == kvb.KVB_OK
     ref = blend.realign(Shape.of(shape, act_bf16=True), np64(k_src), starts)
     e = assert_close_bf16(k_dst[:, :n_ctx].cpu(), ref, "realigned K")
-    assert torch.equal(v_dst[:, :n_ctx].cpu(), v_src), "V must be copied bit-exactly"
+    # bf16 -> fp16 container: the same value (torch rounds to nearest-even like the kernel)
+    assert torch.equal(v_dst[:, :n_ctx].cpu(), v_src.to(torch.float16)), "V must be converted exactly"
+    # and come back unchanged wherever fp16 holds them exactly (zero and |v| >= 2^-14; smaller
+    # magnitudes are fp16 subnormals, rounded to 2^-24)
+    normal = (v_src == 0) | (v_src.float().abs() >= 2.0 ** -14)
+    back = v_dst[:, :n_ctx].cpu().to(torch.bfloat16)
+    assert torch.equal(back[normal], v_src[normal]), "V values must survive the round trip"
+    assert (back[~normal].float() - v_src[~normal].float()).abs().max() <= 2.0 ** -25
     assert torch.count_nonzero(k_dst[:, n_ctx:]) == 0, "rows past n_ctx must be untouched"
     # in place gives the same bits as out of place
     k_in = dev(k_src).clone()
@@ -135,12 +145,21 @@ def test_gather_rmsnorm_qkv_matches_oracle(kvb, shape, m, n_src):
 
 # ------------------------------------------------------------------------------------------ attention
 
-def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
+def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11, tagged=False):
+    """Runs the attention kernel on one case and the oracle on all its rows.  Default inputs:
+    queries scaled for logits of standard deviation 5 (a peaked softmax) against N(0,1) keys;
+    tagged=True: the tagged-key construction of tests/attn_cases.py, where each (row, head)
+    reads essentially one chosen key, so a key range that is off by one key or one tile
+    changes the output completely."""
     cfg = kvb.config(shape)
     m = len(q_rows)
-    q = synth.randn_bf16((m, shape.n_q_heads, shape.head_dim), seed)
-    k = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 1)
-    v = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 2).to(torch.float16)
+    if tagged:
+        q, k, v, _ = tagged_case(n_kv, q_rows, kv_lo, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, seed)
+        v = v.to(torch.float16)
+    else:
+        q = peaked_queries(m, shape.n_q_heads, shape.head_dim, seed)
+        k = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 1)
+        v = synth.randn_bf16((n_kv, shape.n_kv_heads, shape.head_dim), seed + 2).to(torch.float16)
     qi = torch.tensor(q_rows, dtype=torch.int32)
     lo = None if kv_lo is None else torch.tensor(kv_lo, dtype=torch.int32)
     out = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
@@ -149,37 +168,40 @@ def _attn_case(kvb, shape, n_kv, q_rows, kv_lo=None, seed=11):
     torch.cuda.synchronize()
     assert kvb.device_status(ws) == 0
     ref = llama.attention_rows(Shape.of(shape), np64(q), np64(k), np64(v), q_rows, kv_lo)
-    return out.cpu(), ref.reshape(m, -1), float(np.sqrt(np.mean(np64(v) ** 2)))
+    return out.cpu(), ref.reshape(m, -1)
 
 
+@pytest.mark.parametrize("tagged", [False, True])
 @pytest.mark.parametrize("shape,n_kv", [(TINY, 544), (L8B, 3904), (TINY, 1), (L8B, 130), (L8B, 129), (YT, 544),
                                         (Y2, 3904), (Y2, 19), (YT, 1)])
-def test_attention_dense_causal(kvb, shape, n_kv):
-    out, ref, vs = _attn_case(kvb, shape, n_kv, list(range(n_kv)))
-    e = assert_close_rel(out, ref, "dense causal attention", scale=vs)
-    print("attn dense", shape.head_dim, n_kv, e)
+def test_attention_dense_causal(kvb, shape, n_kv, tagged):
+    out, ref = _attn_case(kvb, shape, n_kv, list(range(n_kv)), tagged=tagged)
+    e = assert_attn_close(out, ref, "dense causal attention")
+    print("attn dense", shape.head_dim, n_kv, tagged, e)
 
 
+@pytest.mark.parametrize("tagged", [False, True])
 @pytest.mark.parametrize("shape,n_kv,m", [(TINY, 544, 108), (L8B, 3904, 640), (L8B, 3904, 33), (L8B, 5000, 1),
                                           (TINY, 200, 3), (Y2, 3904, 640), (YT, 544, 37)])
-def test_attention_sparse_rows(kvb, shape, n_kv, m):
+def test_attention_sparse_rows(kvb, shape, n_kv, m, tagged):
     g = np.random.default_rng(m)
     rows = np.sort(g.choice(n_kv, size=m, replace=False))
     rows[-1] = n_kv - 1
-    out, ref, vs = _attn_case(kvb, shape, n_kv, rows.tolist())
-    e = assert_close_rel(out, ref, "sparse-query attention", scale=vs)
-    print("attn sparse", shape.head_dim, n_kv, m, e)
+    out, ref = _attn_case(kvb, shape, n_kv, rows.tolist(), tagged=tagged)
+    e = assert_attn_close(out, ref, "sparse-query attention")
+    print("attn sparse", shape.head_dim, n_kv, m, tagged, e)
 
 
+@pytest.mark.parametrize("tagged", [False, True])
 @pytest.mark.parametrize("shape,starts", [(TINY, [0, 128, 256, 384, 512]), (L8B, [0, 480, 960, 1440]),
                                           (TINY, [0, 5, 140, 141, 300]), (Y2, [0, 480, 960, 1440]),
-                                          (YT, [0, 5, 140, 141, 300])])
-def test_attention_block_diagonal(kvb, shape, starts):
+                                          (YT, [0, 5, 140, 141, 300]), (L8B, [0, 143, 144, 289, 577, 1000])])
+def test_attention_block_diagonal(kvb, shape, starts, tagged):
     n = starts[-1]
     lo = np.concatenate([[starts[c]] * (starts[c + 1] - starts[c]) for c in range(len(starts) - 1)])
-    out, ref, vs = _attn_case(kvb, shape, n, list(range(n)), lo.tolist())
-    e = assert_close_rel(out, ref, "block-diagonal attention", scale=vs)
-    print("attn blockdiag", shape.head_dim, e)
+    out, ref = _attn_case(kvb, shape, n, list(range(n)), lo.tolist(), tagged=tagged)
+    e = assert_attn_close(out, ref, "block-diagonal attention")
+    print("attn blockdiag", shape.head_dim, tagged, e)
 
 
 # ------------------------------------------------------------------------------------------ MLP half
@@ -240,6 +262,106 @@ def test_kv_scatter_skips_rows_outside_the_destination(kvb):
     assert torch.equal(kpad.cpu(), want_k) and torch.equal(vpad.cpu(), want_v)
 
 
+@pytest.mark.parametrize("noalloc", [False, True])
+def test_qkv_indices_outside_their_range_are_reported(kvb, noalloc):
+    """Destinations outside [0, n_kv_rows) write no k/v row and positions outside the RoPE
+    tables rotate by position 0; both set KVB_ERR_INVALID_ARG in the status word, and every
+    other row comes out exactly as in a run with valid indices.  The k/v destination is a
+    view that starts one row into a larger buffer, and the tables hold one row more than
+    the struct declares, so the rows the bad indices name (-1, n_kv_rows, max_pos) are all
+    memory of this test; they must stay untouched."""
+    shape = L8B
+    cfg = kvb.config(shape)
+    lws = kvb.layer_struct({k: dev(v) for k, v in synth.make_layer_weights(shape, 1, seed=6).items()})
+    m, n_rows, max_pos = 8, 40, 30
+    g = torch.Generator().manual_seed(17)
+    x = dev(torch.randn(m, shape.hidden, generator=g))
+    good_dst = torch.tensor([3, 7, 11, 15, 19, 23, 27, 31], dtype=torch.int32)
+    good_pos = torch.tensor([0, 1, 5, 9, 13, 17, 21, 29], dtype=torch.int32)
+    bad_dst = good_dst.clone()
+    bad_dst[2], bad_dst[5] = -1, n_rows                 # rows 2 and 5 must write nothing
+    bad_pos = good_pos.clone()
+    bad_pos[4] = max_pos                                # row 4 is rotated by position 0
+    ref_pos = good_pos.clone()
+    ref_pos[4] = 0
+    rope = kvb.RopeTable(cfg, max_pos + 1)
+    rope.struct.max_pos = max_pos
+
+    def run(dst, pos):
+        q = torch.zeros(m, shape.q_dim, dtype=torch.bfloat16, device="cuda")
+        kbig = torch.zeros(n_rows + 2, shape.kv_dim, dtype=torch.bfloat16, device="cuda")
+        vbig = torch.zeros(n_rows + 2, shape.kv_dim, dtype=torch.float16, device="cuda")
+        kview, vview = kbig[1:n_rows + 1], vbig[1:n_rows + 1]
+        if noalloc:
+            st = torch.zeros(4, dtype=torch.int32, device="cuda")
+            kvb.gather_rmsnorm_qkv_noalloc(cfg, lws, rope, x, None, dev(pos), m, q, kview, vview, dev(dst), st,
+                                           n_kv_rows=n_rows)
+            torch.cuda.synchronize()
+            code = int(st[0])
+        else:
+            ws = kvb.workspace(cfg, m)
+            kvb.gather_rmsnorm_qkv(cfg, lws, rope, x, None, dev(pos), m, q, kview, vview, dev(dst), ws,
+                                   n_kv_rows=n_rows)
+            code = kvb.device_status(ws)
+        return code, q.cpu(), kbig.cpu(), vbig.cpu()
+
+    code, q, kb, vb = run(bad_dst, bad_pos)
+    assert code == kvb.KVB_ERR_INVALID_ARG
+    code_ref, q_ref, kb_ref, vb_ref = run(good_dst, ref_pos)
+    assert code_ref == kvb.KVB_OK
+    assert torch.equal(q, q_ref), "q rows, including the one rotated by position 0"
+    assert torch.count_nonzero(kb[0]) == 0 and torch.count_nonzero(kb[n_rows + 1]) == 0
+    assert torch.count_nonzero(vb[0]) == 0 and torch.count_nonzero(vb[n_rows + 1]) == 0
+    for r in range(m):
+        row = int(good_dst[r]) + 1
+        if r in (2, 5):
+            assert torch.count_nonzero(kb[row]) == 0 and torch.count_nonzero(vb[row]) == 0
+        else:
+            assert torch.equal(kb[row], kb_ref[row]) and torch.equal(vb[row], vb_ref[row]), r
+
+
+def test_realign_reports_v_outside_fp16_range(kvb):
+    """A chunk-cache V value beyond fp16's finite range (|v| > 65504) cannot be held by the
+    blended cache's fp16 containers: the merge writes it as +-65504, keeps NaN as NaN,
+    converts every other value exactly and records KVB_ERR_RANGE; the largest bf16 value
+    that fits (65280) and the smallest normal fp16 magnitude pass without a report."""
+    shape = TINY
+    cfg = kvb.config(shape)
+    L, n_ctx, Hkv, D = 1, 8, shape.n_kv_heads, shape.head_dim
+    starts = dev(torch.tensor([0, 5, 8], dtype=torch.int32))
+    rope = kvb.RopeTable(cfg, n_ctx)
+    k = dev(synth.randn_bf16((L, n_ctx, Hkv, D), 501))
+    v = synth.randn_bf16((L, n_ctx, Hkv, D), 502)
+    v[0, 1, 0, 3] = 65280.0                              # largest bf16 value below fp16's limit
+    v[0, 2, 1, 0] = -(2.0 ** -14)                        # smallest normal fp16 magnitude
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    kd = torch.zeros(L, n_ctx, Hkv, D, dtype=torch.bfloat16, device="cuda")
+    vd = torch.zeros(L, n_ctx, Hkv, D, dtype=torch.float16, device="cuda")
+    kvb.rope_realign(cfg, rope, k, dev(v), kd, vd, 0, L, starts, n_ctx, ws=ws)
+    assert kvb.device_status(ws) == kvb.KVB_OK
+    assert torch.equal(vd.cpu(), v.to(torch.float16))
+    vbad = v.clone()
+    vbad[0, 3, 0, 5] = 65536.0
+    vbad[0, 6, 1, 7] = -1.0e30
+    vbad[0, 7, 0, 0] = float("inf")
+    vbad[0, 4, 1, 1] = float("nan")
+    kvb.rope_realign(cfg, rope, k, dev(vbad), kd, vd, 0, L, starts, n_ctx, ws=ws)
+    assert kvb.device_status(ws) == kvb.KVB_ERR_RANGE
+    got = vd.cpu().float()
+    assert got[0, 3, 0, 5] == 65504.0 and got[0, 6, 1, 7] == -65504.0 and got[0, 7, 0, 0] == 65504.0
+    assert torch.isnan(got[0, 4, 1, 1])
+    want = v.to(torch.float16).float()
+    mask = torch.ones_like(got, dtype=torch.bool)
+    for idx in ((0, 3, 0, 5), (0, 6, 1, 7), (0, 7, 0, 0), (0, 4, 1, 1)):
+        mask[idx] = False
+    assert torch.equal(got[mask], want[mask])
+    # in place (the same memory holds bf16 before and fp16 after) gives the same bits
+    vin = dev(v).clone()
+    kvb.rope_realign(cfg, rope, k, vin, kd, vin, 0, L, starts, n_ctx, ws=ws)
+    assert kvb.device_status(ws) == kvb.KVB_OK
+    assert torch.equal(vin.view(torch.float16).cpu(), v.to(torch.float16))
+
+
 def _tiny_device_model(kvb, pad_embed_rows=0):
     w = synth.make_model(TINY, 0)
     emb = torch.zeros(TINY.vocab + pad_embed_rows, TINY.hidden, dtype=torch.bfloat16, device="cuda")
@@ -279,7 +401,7 @@ def test_forced_selection_outside_the_context_is_reported(kvb):
     rope = kvb.RopeTable(cfg, wl.n_total)
     toks = wl.tokens().cuda()
     kch = torch.zeros(TINY.n_layers, wl.n_ctx, TINY.n_kv_heads, TINY.head_dim, dtype=torch.bfloat16, device="cuda")
-    vch = torch.zeros(kch.shape, dtype=torch.float16, device="cuda")
+    vch = torch.zeros(kch.shape, dtype=torch.bfloat16, device="cuda")
     ck = torch.zeros(TINY.n_layers, wl.n_total, TINY.n_kv_heads, TINY.head_dim, dtype=torch.bfloat16, device="cuda")
     cv = torch.zeros(ck.shape, dtype=torch.float16, device="cuda")
     starts = torch.tensor(wl.chunk_starts(), dtype=torch.int32, device="cuda")

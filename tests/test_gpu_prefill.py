@@ -62,6 +62,7 @@ class Case:
         # floor: float32 accumulation, same bf16 rounding points
         full32 = blend.full_prefill(Shape.of(self.shape, act_bf16=True, accum32=True), self.l64, x0)
         fh32 = llama.rmsnorm(full32["x"][-self.nq:], np64(w["final_norm"]), self.s.rms_eps)
+        self.full_fh32 = fh32
         self.floor = {"fh": errs(fh32, self.full_fh)["mean_abs"]}
         for l in range(self.shape.n_layers):
             self.floor[f"k{l}"] = errs(full32["k"][l], self.full["k"][l])["mean_abs"]
@@ -75,7 +76,7 @@ class Case:
         self.dtoks = self.toks.cuda()
         self.dstarts = torch.tensor(self.starts, dtype=torch.int32, device="cuda")
         self.kch = torch.from_numpy(self.cc["k"]).to(torch.bfloat16).cuda()
-        self.vch = torch.from_numpy(self.cc["v"]).to(torch.bfloat16).to(torch.float16).cuda()
+        self.vch = torch.from_numpy(self.cc["v"]).to(torch.bfloat16).cuda()       # chunk-cache format
         self.ws = kvb.workspace(self.cfg, self.N)
 
     def mean_bar(self, key, scale=1.0):
@@ -118,6 +119,8 @@ def test_full_prefill_matches_oracle(kvb, case):
     assert kvb.device_status(case.ws) == 0
     e = case.check_fh(fh.cpu(), case.full_fh, "final hidden (dense prefill)")
     e64 = case.fp64_gap(fh.cpu(), case.full_fh64, "final hidden (dense prefill)")
+    e32 = errs(fh.cpu(), case.full_fh32)     # the fp32-accumulation oracle: reported beside the reference
+    print("full prefill", case.wl.name, "vs fp32-accumulation oracle", e32)
     for l in range(case.shape.n_layers):
         case.check_cache(ck[l].cpu(), case.full["k"][l], f"k{l}", f"layer {l} K")
         case.check_cache(cv[l].cpu(), case.full["v"][l], f"v{l}", f"layer {l} V")
