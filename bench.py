@@ -69,7 +69,7 @@ def parse():
     ap.add_argument("--sweep", action="store_true",
                     help="64k-context sweep: r x chunk size, per-kernel times (prints one JSON line per point)")
     ap.add_argument("--kernel", default=None,
-                    choices=["attn", "dense", "gemm", "realign", "decode_attn", "decode_step"],
+                    choices=["attn", "dense", "gemm", "realign", "decode_attn", "decode_step", "topk", "hkvd"],
                     help="time one kernel of the library on a seeded synthetic Llama-3.1-8B-shaped case "
                          "(for ncu captures); prints one JSON line")
     ap.add_argument("--m", type=int, default=18713, help="--kernel attn / gemm: query rows")
@@ -696,6 +696,19 @@ def run_kernel(args) -> None:
             kvb.decode_step(cfgl, model, rope, kc, vc, lm, tokens, pos, n_kv, ws=ws)
         wb = args.layers * 2.0 * (shp.qkv_dim * H + H * shp.q_dim + 3 * H * F) + shp.vocab * H * 2.0
         out.update(bytes=wb + args.layers * float(n_kv) * Hkv * D * 4, layers=args.layers, n_kv=n_kv)
+    elif args.kernel in ("topk", "hkvd"):
+        # HKVD selection over --n-ctx context rows at r = 0.15: the deviation over the 1,024
+        # key entries of a row, then the top-k (topk: 8 entries per row, so that the time is
+        # the top-k's)
+        n_ctx = args.n_ctx
+        kvd = 8 if args.kernel == "topk" else Hkv * D
+        kf = torch.randn(n_ctx, kvd, generator=g, device=dev).to(torch.bfloat16)
+        kc = torch.randn(n_ctx, kvd, generator=g, device=dev).to(torch.bfloat16)
+        kk = int(0.15 * n_ctx)
+        sel = torch.empty(kk, dtype=torch.int32, device=dev)
+        dv = torch.empty(n_ctx, dtype=torch.float32, device=dev)
+        fn = lambda: kvb.hkvd_select(kf, kc, kk, sel_out=sel, dev_out=dv)
+        out.update(n_ctx=n_ctx, k=kk, kv_dim=kvd, bytes=4.0 * n_ctx * kvd)
     else:
         L, n_ctx = args.layers, args.n_ctx
         ks = torch.randn(L, n_ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)

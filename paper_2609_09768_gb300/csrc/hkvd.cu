@@ -6,7 +6,13 @@
 // 8-bit passes narrow the k-th largest key with warp-aggregated shared-memory
 // histograms, then an ordered compaction writes the selected indices in
 // ascending order, taking keys equal to the threshold from the lowest index up.
-// One CTA of 1024 threads; the deviations stay in L2 between passes.
+// It runs on one thread-block cluster of 8 CTAs x 1024 threads: each CTA owns a
+// contiguous eighth of the keys (up to 16 per thread, held in registers for the
+// whole select), the CTAs' histograms are summed through distributed shared memory
+// after every pass (each CTA reaches the same digit), and the compaction takes its
+// output offset from the counts of the CTAs before it.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -69,6 +75,102 @@ __device__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_sums, uint32
     return before;
 }
 
+constexpr int TK_CTAS = 8, TK_KPT = 16;
+constexpr int64_t TK_CLUSTER_MAX = (int64_t)TK_CTAS * TOPK_THREADS * TK_KPT;   // 131,072 keys
+
+// warp-aggregated histogram increment for the keys whose bits above `shift + 8` match
+KVB_DEV void hist_add(uint32_t* hist, uint32_t key, uint32_t mask, uint32_t prefix, int shift) {
+    const bool in = (key & mask) == prefix;
+    const uint32_t act = __activemask();
+    const uint32_t want = __ballot_sync(act, in);
+    if (in) {
+        const uint32_t d = (key >> shift) & 255u;
+        const uint32_t peers = __match_any_sync(want, d);
+        if ((threadIdx.x & 31) == (__ffs(peers) - 1)) atomicAdd(&hist[d], __popc(peers));
+    }
+}
+
+// Exact top-k of n <= TK_CLUSTER_MAX keys on one cluster of TK_CTAS CTAs.
+__global__ void __cluster_dims__(TK_CTAS, 1, 1) __launch_bounds__(TOPK_THREADS, 1)
+topk_cluster_kernel(const float* __restrict__ dev, int64_t n, int64_t k, int32_t* __restrict__ sel) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    __shared__ uint32_t hist[256];
+    __shared__ uint32_t tot[256];
+    __shared__ uint32_t warp_sums[32];
+    __shared__ uint32_t s_digit, s_remaining;
+    __shared__ uint32_t cnt[2];               // this CTA's keys above / equal to the threshold
+    const int tid = threadIdx.x;
+    // this thread's keys: indices [tbeg, tbeg + nk), contiguous, so the compaction keeps index order
+    const int64_t tbeg = (int64_t)rank * TOPK_THREADS * TK_KPT + (int64_t)tid * TK_KPT;
+    const int nk = (int)max((int64_t)0, min((int64_t)TK_KPT, n - tbeg));
+    if (k <= 0) return;                       // k and n are the same for every CTA of the cluster
+    if (k >= n) {
+        for (int u = 0; u < nk; ++u) sel[tbeg + u] = (int32_t)(tbeg + u);
+        return;
+    }
+    uint32_t key[TK_KPT];
+#pragma unroll
+    for (int u = 0; u < TK_KPT; ++u) key[u] = u < nk ? __float_as_uint(__ldg(dev + tbeg + u)) : 0u;
+    uint32_t prefix = 0, mask = 0, remaining = (uint32_t)k;
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        if (tid < 256) hist[tid] = 0;
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < TK_KPT; ++u)
+            if (u < nk) hist_add(hist, key[u], mask, prefix, shift);
+        cluster.sync();                       // every CTA's histogram is complete
+        if (tid < 256) {
+            uint32_t sum = 0;
+#pragma unroll
+            for (int r = 0; r < TK_CTAS; ++r) sum += *cluster.map_shared_rank(&hist[tid], r);
+            tot[tid] = sum;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            uint32_t cum = 0;
+            for (int d = 255; d >= 0; --d) {
+                if (cum + tot[d] >= remaining) { s_digit = (uint32_t)d; s_remaining = remaining - cum; break; }
+                cum += tot[d];
+            }
+        }
+        __syncthreads();
+        prefix |= s_digit << shift;
+        mask |= 255u << shift;
+        remaining = s_remaining;
+        cluster.sync();                       // no CTA clears its histogram while another still reads it
+    }
+    // threshold key `prefix`: take every key above it and the first `remaining` equal ones
+    uint32_t gt = 0, eq = 0;
+#pragma unroll
+    for (int u = 0; u < TK_KPT; ++u)
+        if (u < nk) { gt += key[u] > prefix; eq += key[u] == prefix; }
+    uint32_t gt_tot, eq_tot;
+    const uint32_t gt_before = block_exclusive_scan(gt, warp_sums, &gt_tot);
+    const uint32_t eq_before = block_exclusive_scan(eq, warp_sums, &eq_tot);
+    if (tid == 0) { cnt[0] = gt_tot; cnt[1] = eq_tot; }
+    cluster.sync();
+    uint32_t gt_prev = 0, eq_prev = 0;        // counts of the CTAs holding lower indices
+    for (int r = 0; r < rank; ++r) {
+        gt_prev += *cluster.map_shared_rank(&cnt[0], r);
+        eq_prev += *cluster.map_shared_rank(&cnt[1], r);
+    }
+    uint32_t eq_seen = eq_prev + eq_before;
+    uint32_t out = gt_prev + gt_before + (eq_seen < remaining ? eq_seen : remaining);
+#pragma unroll
+    for (int u = 0; u < TK_KPT; ++u) {
+        if (u < nk) {
+            bool take = key[u] > prefix;
+            if (key[u] == prefix) { take = eq_seen < remaining; ++eq_seen; }
+            if (take) sel[out++] = (int32_t)(tbeg + u);
+        }
+    }
+    cluster.sync();                           // keep this CTA's counts readable until every CTA has read them
+}
+
+// One CTA for any n (the cluster kernel above covers n <= TK_CLUSTER_MAX).
 __global__ void __launch_bounds__(TOPK_THREADS)
 topk_kernel(const float* __restrict__ dev, int64_t n, int64_t k, int32_t* __restrict__ sel) {
     __shared__ uint32_t hist[256];
@@ -179,7 +281,10 @@ kvb_status launch_hkvd(const uint16_t* k_fresh, int64_t ld_fresh, const uint16_t
     count_launch();
     kvb_status s = cuda_ok(cudaGetLastError(), "deviation launch");
     if (s != KVB_OK || k <= 0) return s;
-    topk_kernel<<<1, TOPK_THREADS, 0, st>>>(dev_out, n_ctx, k, sel_out);
+    if (n_ctx <= TK_CLUSTER_MAX)
+        topk_cluster_kernel<<<TK_CTAS, TOPK_THREADS, 0, st>>>(dev_out, n_ctx, k, sel_out);
+    else
+        topk_kernel<<<1, TOPK_THREADS, 0, st>>>(dev_out, n_ctx, k, sel_out);
     count_launch();
     return cuda_ok(cudaGetLastError(), "top-k launch");
 }

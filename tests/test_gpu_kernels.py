@@ -73,7 +73,7 @@ def test_realign_matches_oracle(kvb, shape, starts):
 
 @pytest.mark.parametrize("n,kv_dim,k", [
     (512, 128, 76), (3840, 1024, 576), (1000, 64, 333), (17, 128, 0), (17, 128, 17), (1, 128, 1),
-    (123904, 1024, 18585), (5000, 1024, 1),
+    (123904, 1024, 18585), (5000, 1024, 1), (131072, 128, 20000), (131073, 128, 20000), (200000, 128, 30000),
 ])
 def test_hkvd_select_matches_oracle(kvb, n, kv_dim, k):
     kf = synth.randn_bf16((n, kv_dim), 201)
@@ -93,6 +93,20 @@ def test_hkvd_select_matches_oracle(kvb, n, kv_dim, k):
     assert np.all(np.diff(s) > 0), "indices must be ascending and distinct"
     nd = check_selection(s, dref, k)
     print("hkvd", n, k, "dev err", e["max_abs"], "differing (near-tie) indices", nd)
+
+
+@pytest.mark.parametrize("n", [123904, 131072, 200000])
+def test_hkvd_all_equal_deviations_take_the_lowest_indices(kvb, n):
+    """Every deviation equal: the top k are exactly indices 0..k-1, also where the k-th
+    falls on the boundary between the key ranges of two CTAs of the select's cluster
+    (16,384 keys each) and on the last key."""
+    kv_dim = 8
+    kf = torch.zeros(n, kv_dim, dtype=torch.bfloat16)
+    kc = kf.clone()
+    kc[:, 3] = 0.5
+    for k in (1, 16383, 16384, 16385, 65536, n - 1, n):
+        sel, _ = kvb.hkvd_select(dev(kf), dev(kc), k)
+        assert torch.equal(sel.cpu(), torch.arange(k, dtype=torch.int32)), k
 
 
 def test_hkvd_exact_ties_take_lowest_index(kvb):
