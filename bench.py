@@ -64,7 +64,8 @@ def parse():
     ap.add_argument("--r1-steps", type=int, default=1, help="timed steps of the r = 1.0 comparator (0: skip)")
     ap.add_argument("--e2e-steps", type=int, default=2, help="timed end-to-end steps (0: skip)")
     ap.add_argument("--decode-steps", type=int, default=16, help="greedy decode steps timed after the prefill (0: skip)")
-    ap.add_argument("--cpu-rows", type=int, default=512, help="rows in the oracle's timed sample")
+    ap.add_argument("--cpu-rows", type=int, default=128,
+                    help="rows in the oracle's timed sample (the same for the cpu_baseline leg and the reference arm)")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--sweep", action="store_true",
                     help="64k-context sweep: r x chunk size, per-kernel times (prints one JSON line per point)")
@@ -158,10 +159,30 @@ class Clocks:
 
 # ------------------------------------------------------------------------------------ oracle (CPU) leg
 
+ORACLE_BLOCK = 256     # rows per block of the oracle's attention (oracle.llama.attention_rows)
+
+
+def oracle_attention_work(hi, lo=None, block: int = ORACLE_BLOCK) -> float:
+    """The oracle's attention work for a set of rows, in (row, key) pairs: it takes the rows in
+    blocks of `block` consecutive rows and scores each block against the union of its rows' key
+    ranges [min lo, max hi], so its cost is the sum over blocks of rows x keys in that union."""
+    import numpy as np
+    hi = np.asarray(hi, dtype=np.int64)
+    lo = np.zeros_like(hi) if lo is None else np.asarray(lo, dtype=np.int64)
+    w = 0.0
+    for b0 in range(0, len(hi), block):
+        h, l = hi[b0:b0 + block], lo[b0:b0 + block]
+        w += float(len(h)) * float(h.max() - l.min() + 1)
+    return w
+
+
 class OracleSample:
     """A bounded sample of the workload for the CPU oracle: one selective decoder layer
     over `n_rows` rows spread uniformly over the context, attending a float64 cache of
-    the full request length.  Inputs are drawn once; run() times the oracle call."""
+    the full request length.  Inputs are drawn once; run() times the oracle's steps in two
+    parts: the per-row part (RMSNorm, q/k/v projection and RoPE, O-projection, RMSNorm and
+    SwiGLU MLP), and the attention, whose cost per row depends on the key range the
+    oracle scores it against."""
 
     def __init__(self, wl, n_rows: int, seed: int = 0):
         import numpy as np
@@ -178,12 +199,21 @@ class OracleSample:
         self.rows = np.sort(rng.choice(wl.n_ctx, size=n_rows, replace=False))
         self.x = rng.standard_normal((n_rows, shape.hidden))
         self.n_rows = n_rows
+        self.work = oracle_attention_work(self.rows)
 
-    def run(self) -> float:
+    def run(self):
+        """(seconds of the per-row part, seconds of the attention) for one oracle layer."""
         from oracle import llama
         t0 = time.perf_counter()
-        llama.layer_rows(self.s, self.lw, self.x, self.rows, self.rows, self.kc, self.vc)
-        return time.perf_counter() - t0
+        q, k, v = llama.qkv_rows(self.s, self.lw, self.x, self.rows)
+        t1 = time.perf_counter()
+        self.kc[self.rows] = k
+        self.vc[self.rows] = v
+        a = llama.act(self.s, llama.attention_rows(self.s, q, self.kc, self.vc, self.rows))
+        t2 = time.perf_counter()
+        llama.attn_out_mlp(self.s, self.lw, self.x, a.reshape(a.shape[0], -1))
+        t3 = time.perf_counter()
+        return (t1 - t0) + (t3 - t2), t2 - t1
 
 
 def cpu_cores() -> int:
@@ -193,11 +223,21 @@ def cpu_cores() -> int:
         return os.cpu_count() or 1
 
 
-def oracle_ttft_ms(wl, seconds: float, rows: int, k: int) -> float:
-    """Scale a sample to the prefill: layer 0 over all N rows plus (L-1) layers over m rows."""
-    m = k + wl.n_query
-    row_layers = wl.n_total + (wl.shape.n_layers - 1) * m
-    return seconds / rows * row_layers * 1e3
+def oracle_ttft_ms(wl, smp: "OracleSample", t_rows: float, t_attn: float, k: int, sel=None) -> float:
+    """The oracle's prefill time from one timed sample layer:
+         per-row part:  t_rows / sample rows  x  (N + (L - 1) m) row-layers
+         attention:     t_attn / sample work  x  (work of layer 0 + (L - 1) x work of a selective layer)
+    with the work of oracle_attention_work: layer 0 scores all N rows causally, a selective
+    layer the m = k + n_query recomputed rows (the selected context rows `sel`, or k rows
+    spread uniformly when they are not known, then the query rows) over [0, own row]."""
+    import numpy as np
+    N, L, nq = wl.n_total, wl.shape.n_layers, wl.n_query
+    m = k + nq
+    if sel is None:
+        sel = np.linspace(0, wl.n_ctx - 1, num=k).round().astype(np.int64) if k else np.zeros(0, np.int64)
+    rows_sel = np.concatenate([np.sort(np.asarray(sel, dtype=np.int64)), np.arange(wl.n_ctx, N)])
+    work = oracle_attention_work(np.arange(N)) + (L - 1) * oracle_attention_work(rows_sel)
+    return (t_rows / smp.n_rows * (N + (L - 1) * m) + t_attn / smp.work * work) * 1e3
 
 
 def run_reference(args, wl, rank: int, world: int) -> None:
@@ -207,16 +247,17 @@ def run_reference(args, wl, rank: int, world: int) -> None:
     from oracle import blend
     r = wl.r if args.r is None else args.r
     k = blend.num_selected(r, wl.n_ctx)
-    rows = max(16, min(64, args.cpu_rows))
+    rows = max(16, min(256, args.cpu_rows))
     smp = OracleSample(wl, rows)
     for _ in range(args.warmup):
         smp.run()
     vals = []
     for _ in range(args.steps):
-        vals.append(oracle_ttft_ms(wl, smp.run(), rows, k))
+        vals.append(oracle_ttft_ms(wl, smp, *smp.run(), k))
     v = statistics.mean(vals)
     sample = (f"oracle selective layer on {rows} of {k + wl.n_query} recomputed rows (uniform over the context) "
-              f"attending a {wl.n_total}-row cache, per step; scaled by (N + (L-1) m) row-layers")
+              f"attending a {wl.n_total}-row cache, per step; per-row part scaled by (N + (L-1) m) row-layers, "
+              f"attention by the oracle's (row, key) block work of the whole prefill (extrapolated)")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "ms", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(v, 3), "higher_is_better": False,
@@ -367,20 +408,33 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         hf = torch.empty(fh.shape, dtype=fh.dtype, pin_memory=True)
         htok = torch.empty(tok.shape, dtype=tok.dtype, pin_memory=True)
         hk.copy_(kch); hv.copy_(vch); ht.copy_(toks)
+        torch.cuda.synchronize()
+        # the bare host->device copy of the same caches before any e2e step, for reference
+        kd = torch.empty_like(kch)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(); kd.copy_(hk, non_blocking=True); b.record()
+        torch.cuda.synchronize()
+        h2d_k_ms = a.elapsed_time(b)
+        del kd
         td = torch.empty_like(toks)
         wsp = torch.zeros(kvb.workspace_size_pipelined(cfg, N, n_ctx), dtype=torch.uint8, device=dev)
         cs = torch.cuda.Stream(device=dev)
         torch.cuda.synchronize()
 
-        def e2e_step():
+        e2e_t = []
+
+        def e2e_step(timings=False):
             td.copy_(ht, non_blocking=True)
-            kvb.selective_prefill_host(cfg, model, rope, hk, hv, ck, cv, td, dstarts, n_ctx, nq, r, 1,
-                                       copy_stream=cs, final_hidden=fh, sel_out=sel, ws=wsp)
+            t = kvb.selective_prefill_host(cfg, model, rope, hk, hv, ck, cv, td, dstarts, n_ctx, nq, r, 1,
+                                           copy_stream=cs, final_hidden=fh, sel_out=sel, ws=wsp,
+                                           timings=timings)[2]
+            if t:
+                e2e_t.append(t)
             kvb.lm_head_argmax(cfg, lm, fh[nq - 1:], tokens=tok, ws=lm_ws)
             hf.copy_(fh, non_blocking=True)
             htok.copy_(tok, non_blocking=True)
 
-        e2e_step()
+        e2e_step(timings=True)           # untimed: its stage times show where the ingest waits
         torch.cuda.synchronize()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
@@ -397,7 +451,10 @@ def run_ours(args, wl, rank: int, world: int) -> None:
         h2d = hk.numel() * 2 + hv.numel() * 2 + ht.numel() * 4
         e2e = {"value": round(e2e_ms, 3), "unit": "ms", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(hf.numel() * 4 + htok.numel() * 4), "path": "kvb_selective_prefill_host (layer-wise ingest)",
-               "bare_h2d_ms": round(h2d_ms, 2), "bare_h2d_gbs": round(h2d / (h2d_ms * 1e-3) / 1e9, 1)}
+               "bare_h2d_ms": round(h2d_ms, 2), "bare_h2d_gbs": round(h2d / (h2d_ms * 1e-3) / 1e9, 1),
+               "bare_h2d_k_before_gbs": round(hk.numel() * 2 / (h2d_k_ms * 1e-3) / 1e9, 1),
+               "stages_ms_untimed_step": {k_: round(v_, 3) for k_, v_ in e2e_t[0].items() if k_.endswith("_ms")}
+               if e2e_t else None}
         del hk, hv, kd, wsp
 
     # greedy decode after the prefill (first token already decoded by the step): n_dec steps
@@ -459,11 +516,16 @@ def run_ours(args, wl, rank: int, world: int) -> None:
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        n = args.cpu_rows
-        sec = OracleSample(wl, n).run()
-        cpu = {"value": round(oracle_ttft_ms(wl, sec, n, k), 1), "unit": "ms", "cores": cpu_cores(), "kind": "oracle",
+        n = max(16, min(256, args.cpu_rows))
+        smp = OracleSample(wl, n)
+        t_rows, t_attn = smp.run()
+        sel_np = sel[:k].cpu().numpy() if k > 0 else None
+        cpu = {"value": round(oracle_ttft_ms(wl, smp, t_rows, t_attn, k, sel_np), 1), "unit": "ms",
+               "cores": cpu_cores(), "kind": "oracle",
                "sample": (f"oracle selective layer on {n} of {m} recomputed rows (uniform over the context) "
-                          f"attending a {N}-row float64 cache, {sec:.1f} s; scaled by (N + (L-1) m) row-layers "
+                          f"attending a {N}-row float64 cache: {t_rows:.1f} s per-row part + {t_attn:.1f} s "
+                          f"attention; per-row part scaled by (N + (L-1) m) row-layers, attention by the oracle's "
+                          f"(row, key) block work of the whole prefill with the selection this run made "
                           f"(extrapolated)")}
 
     if rank == 0:
