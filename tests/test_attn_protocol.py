@@ -21,7 +21,9 @@ runs out, sets the CTA's abort flag (every later incomplete wait then returns at
 
 Each run checks: every actor finishes (no deadlock, in particular at the P barrier); no
 warp arrives twice in one phase of the named barrier; no parity wait ever finds its
-barrier two phases ahead (which would make the hardware answer wrongly); and, in runs
+barrier two phases ahead, nor asks for a phase while the one before it is still open
+(either would make the hardware answer wrongly: a parity wait cannot tell phase k from
+k - 2); and, in runs
 where no wait runs out, the data hazards are ordered: a slot is reloaded only after the
 P.V that read it, S_j runs only after K_j landed, P.V_j only after all four warps wrote
 P_j, S_{j+2} only after P.V_j read P_j from the same buffer, and O is rescaled only when
@@ -85,6 +87,8 @@ class Protocol:
         c = self.phases(name, idx)
         if c - phase >= 2:
             self.errors.append(f"{name}[{idx}] two phases past the awaited phase {phase} (c = {c})")
+        if c < phase:
+            self.errors.append(f"{name}[{idx}] asked for phase {phase} while phase {c} is still open")
         return (c & 1) != parity
 
     def issue(self, kind, j=None, commit=None):
@@ -287,3 +291,25 @@ def test_model_catches_a_slot_reloaded_too_early():
                 self.events.append((self.t + 5, land))
     with pytest.raises(AssertionError, match="reloaded|two phases past"):
         Eager(12, 0).run()
+
+
+def test_model_catches_a_wait_on_a_phase_not_yet_reached():
+    """A producer that frees slot j % 3 by waiting for S_{j-1} (issued after P.V_{j-3}, so
+    done after it in a single in-order pipe) on the double-buffered s_full barrier asks,
+    at tiles 3 and 4, for a phase the barrier has not reached while the one before is still
+    open; the hardware answers such a parity wait at once.  The model flags it."""
+    class WaitsOnS(Protocol):
+        def producer(self):
+            for j in range(self.n):
+                st = j % STAGES
+                if j >= STAGES:
+                    ok = yield ("wait", "s_full", (j - 1) & 1, ((j - 1) >> 1) & 1, (j - 1) >> 1)
+                    if not ok:
+                        break
+
+                def land(j=j, st=st):
+                    self.done["kv"].add(j)
+                    self.complete("kv_full", st)
+                self.events.append((self.t + 5, land))
+    with pytest.raises(AssertionError, match="still open"):
+        WaitsOnS(12, 0).run()
