@@ -13,25 +13,32 @@
 // needs the whole shared-memory bandwidth on its own, before the TMA writes.
 // Key tiles are 144 rows: the widest that leaves room in the 512 TMEM columns for two S
 // buffers, O and Q while three K/V stages (216 KB) fit in shared memory; every tile's
-// barrier waits and commits on the issuing thread then cover 1,152 cycles of MMAs
-// instead of 1,024 with 128-key tiles.
+// barrier waits and commits then cover 1,152 cycles of MMAs instead of 1,024 with
+// 128-key tiles.
 // TMEM columns: S buffers [0, 144) and [160, 304) (P_j is written over the first 72
 // columns of S_j's buffer), O [320, 448), Q [448, 512).
+//
+// The MMAs are issued by two threads.  The tensor pipe's instruction queue is shallow,
+// so a thread that issues an MMA waits for roughly its execution, and every mbarrier
+// wait and commit on an issuing thread leaves the pipe idle for its duration; with two
+// issuers one thread's waits and commits overlap the other's MMAs.
 //
 // Pipeline per key tile j (144 keys):
 //   TMA warp   : K_j and V_j together into a 3-deep ring (128-byte swizzle); slot
 //                j % 3 is reused once P.V of the tile that held it has completed
-//   MMA thread : S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=144, K=16 steps,
-//                A = Q from TMEM); after the softmax of tile j-1 (a named barrier that
-//                the softmax warps arrive on and the MMA warp blocks on),
-//                O += P_{j-1} V_{j-1} (A = P from TMEM, V an MN-major operand)
+//   S issuer   : waits for K_j, then (j >= 2) for P.V_{j-2}, which read P_{j-2} from the
+//                TMEM buffer S_j overwrites (the two issuers' MMAs are not ordered with
+//                each other); S_j = Q K_j^T into TMEM buffer j%2 (M=128, N=144, K=16
+//                steps, A = Q from TMEM)
+//   P.V issuer : waits for V_j, then for the softmax of tile j (a named barrier that the
+//                softmax warps and this warp pass); O += P_j V_j (A = P from TMEM, V an
+//                MN-major operand)
 //   4 softmax warps (thread = row): load the row's Q into TMEM once; per tile
 //                read S_j from TMEM, mask, online softmax with a lazily updated
 //                running max (O is rescaled only when the max grows by more than
 //                2^8, after P.V_{j-1} is done), write P_j over S_j.  The buffer's
-//                previous P (tile j-2) was read by P.V_{j-2}, which ran before S_j
-//                (MMAs complete in issue order), so the common path waits for
-//                nothing but S_j.
+//                previous P (tile j-2) was read by P.V_{j-2} before S_j was issued,
+//                so the common path waits for nothing but S_j.
 // Lazy rescaling keeps the result exact: every term uses the same reference max
 // as the running sum it is divided by.
 // Precision: Q.K^T runs on bf16 operands; P.V runs on fp16 operands - the
@@ -46,16 +53,16 @@
 namespace kvb {
 namespace {
 
-constexpr int THREADS = 192;
+constexpr int THREADS = 224;                 // producer, S issuer, 4 softmax warps, P.V issuer
+constexpr int WARP_PV = 6;
 constexpr int KT_ROWS = 144;                 // keys per tile
 constexpr int STAGES = 3;                    // K and V ring depth
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t COL_S = 0, S_STRIDE = 160, COL_O = 320, COL_Q = 448;   // S buffers 32-column aligned
-// P_j written -> MMA warp: one named barrier that the 4 softmax warps and the MMA warp
-// all pass with bar.sync once per key tile, in lockstep, on every path (also after a
-// failed wait), so each phase completes and no warp can arrive twice in one phase.  The
-// softmax warps lose nothing by blocking there: the S MMA they wait for next was issued
-// before the MMA warp reached the barrier.
+// P_j written -> P.V issuer: one named barrier that the 4 softmax warps and the P.V
+// issuer's warp all pass with bar.sync once per key tile, in lockstep, on every path
+// (also after a failed wait), so each phase completes and no warp can arrive twice in
+// one phase.
 constexpr uint32_t BAR_P = 1, BAR_P_COUNT = 5 * 32;
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr float P_SHIFT_LOG2 = 7.0f;         // P scaled by 2^7: max 2^(8+7) < 65504
@@ -78,19 +85,20 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
-    // Every wait of the MMA thread and every tcgen05.commit costs the tensor pipe tens to
-    // hundreds of cycles, so each key tile uses two of each: kv_full (K_j and V_j
-    // landed, an mbarrier) and P_{j-1} written (the named barrier BAR_P) for the MMA
-    // warp; s_full (S_j done) and pv_done (P.V_i done) as commits.  P.V_i done also
-    // frees slot i % STAGES for the producer (P_i was written after S_i had been read)
-    // and tells a softmax that must rescale O that the accumulation it rescales is
-    // complete.
+    // Barriers per key tile: kv_full (K_j and V_j landed; waited by both issuers), P_j
+    // written (the named barrier BAR_P), s_full (S_j done) and pv_done (P.V_i done) as
+    // commits.  P.V_i done frees slot i % STAGES for the producer (P_i was written after
+    // S_i had been read), frees S buffer i % 2 for S_{i+2}, and tells a softmax that must
+    // rescale O that the accumulation it rescales is complete.  Every waiter on pv_done
+    // or kv_full either waits for each phase in turn or cannot be more than one phase
+    // behind, so no parity wait meets a barrier two phases away.
     uint64_t* q_ready = bars + 0;                // Q rows stored into TMEM (4 warps)
     uint64_t* kv_full = bars + 1;                // [STAGES]: K_j and V_j in slot j % STAGES
     uint64_t* s_full = kv_full + STAGES;         // [2]: S_j done, phase j/2 of s_full[j % 2]
     uint64_t* pv_done = s_full + 2;              // [STAGES]: P.V_i done, phase i/3 of pv_done[i % 3]
-    uint64_t* drain = pv_done + STAGES;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* drain = pv_done + STAGES;          // P.V issuer's MMAs drained
+    uint64_t* drain_s = drain + 1;               // S issuer's MMAs drained
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_s + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* red = reinterpret_cast<int*>(tmem_slot + 2);   // lo_min, hi_max, hi_min, lo_max
 
@@ -109,6 +117,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
         }
         for (int b = 0; b < 2; ++b) mbar_init(&s_full[b], 1);
         mbar_init(drain, 1);
+        mbar_init(drain_s, 1);
         *abort_flag = 0;
         red[0] = INT_MAX; red[1] = -1; red[2] = INT_MAX; red[3] = -1;
         fence_mbar_init();
@@ -121,7 +130,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     const int L = (int)(quarter * 32 + lane);
     const int64_t row = r0 + L / G;
     const int head = g * G + L % G;
-    const bool valid = warp >= 2 && L < RPB * G && row < p.m;
+    const bool valid = warp >= 2 && warp < WARP_PV && L < RPB * G && row < p.m;
     int hi = -1, lo = 0;
     if (valid) {
         hi = p.q_idx[row];
@@ -170,56 +179,60 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
             }
         }
     } else if (warp == 1) {
-        if (n_tiles > 0) {
-            // ------------------------------------------------ MMA issuer (lane 0; the whole warp
-            // takes part in the named-barrier waits for P)
+        if (n_tiles > 0 && lane == 0) {
+            // ------------------------------------------------ S issuer: S_j = Q K_j^T
             constexpr uint32_t IDESC_S = idesc_bf16(128, KT_ROWS, false);
-            constexpr uint32_t IDESC_O = idesc_f16kind(128, D, true, false);   // fp16 P and V
-            const uint32_t k0 = smem_u32(sK), v0 = smem_u32(sV);
-            bool ok = true;
-            if (lane == 0) ok = mbar_wait(q_ready, 0, abort_flag, p.status);
+            const uint32_t k0 = smem_u32(sK);
+            bool ok = mbar_wait(q_ready, 0, abort_flag, p.status);
             tc_fence_after();
-            for (int j = 0; j <= n_tiles; ++j) {
-                if (j < n_tiles && lane == 0 && ok) {
-                    const int b = j & 1, st = j % STAGES;
-                    // S buffer b last held S_{j-2}: the softmax read it before writing P_{j-2},
-                    // which P.V_{j-2} (issued before this MMA, so executed before it) consumed
-                    ok = mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status);
-                    if (ok) {
-                        tc_fence_after();
-                        // descriptor built once per tile; constant steps inside the unrolled loop keep
-                        // the issuing thread ahead of the MMAs
-                        const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
-                        const uint32_t sd = tmem_base + COL_S + b * S_STRIDE, qa = tmem_base + COL_Q;
+            for (int j = 0; j < n_tiles && ok; ++j) {
+                const int b = j & 1, st = j % STAGES;
+                // S buffer b last held P_{j-2}: wait until P.V_{j-2} (another thread's MMAs, so
+                // not ordered with these) has read it.  Waits on pv_done are contiguous here
+                // (tiles 0, 1, 2, ...), so each finds its barrier in the phase it asks for.
+                // K_j first (it has almost always landed), so that nothing but the issue follows
+                // the wait for P.V_{j-2}
+                ok = mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status);
+                if (ok && j >= 2)
+                    ok = mbar_wait(&pv_done[(j - 2) % STAGES], (uint32_t)((j - 2) / STAGES) & 1, abort_flag, p.status);
+                if (!ok) break;
+                tc_fence_after();
+                const uint64_t kd = sdesc_sw128(k0 + st * S::KV_BYTES, 16, 1024);
+                const uint32_t sd = tmem_base + COL_S + b * S_STRIDE, qa = tmem_base + COL_Q;
 #pragma unroll
-                        for (int kk = 0; kk < D / 16; ++kk) {
-                            // A = Q from TMEM: 16 head dims = 8 columns of bf16 pairs
-                            mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32),
-                                       IDESC_S, kk > 0 ? 1u : 0u);
-                        }
-                        mma_commit(&s_full[b]);
-                    }
-                }
-                if (j >= 1) {
-                    const int i = j - 1, st = i % STAGES;
-                    // P_i written by all four softmax warps: a blocking hardware barrier, not a
-                    // polling loop, so the issuing thread takes no data-dependent branch here
-                    __syncwarp();
-                    named_bar_sync(BAR_P, BAR_P_COUNT);
-                    if (lane == 0 && ok) {
-                        tc_fence_after();
-                        // V_i landed with K_i (kv_full waited in iteration i)
-                        const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
-                        // P_i sits in the first half of its own S buffer
-                        const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (i & 1) * S_STRIDE;
-                        mma_f16_ts(od, pa, vd, IDESC_O, i > 0 ? 1u : 0u);
+                for (int kk = 0; kk < D / 16; ++kk)
+                    mma_f16_ts(sd, qa + kk * 8, sdesc_add(kd, (kk >> 2) * S::CHUNK + (kk & 3) * 32),
+                               IDESC_S, kk > 0 ? 1u : 0u);
+                mma_commit(&s_full[b]);
+            }
+            mma_commit(drain_s);
+            const uint64_t t0 = globaltimer();
+            while (!mbar_try_wait(drain_s, 0) && globaltimer() - t0 < kWaitLimitNs) {}
+        }
+        __syncwarp();
+    } else if (warp == WARP_PV) {
+        if (n_tiles > 0) {
+            // ------------------------------------------------ P.V issuer: O += P_j V_j (lane 0; the
+            // whole warp passes the named barrier for P)
+            constexpr uint32_t IDESC_O = idesc_f16kind(128, D, true, false);   // fp16 P and V
+            const uint32_t v0 = smem_u32(sV);
+            bool ok = true;
+            for (int j = 0; j < n_tiles; ++j) {
+                const int st = j % STAGES;
+                // V_j landed (waited before the barrier, while the softmax works; the phase
+                // cannot move on before this thread commits P.V_j)
+                if (lane == 0 && ok) ok = mbar_wait(&kv_full[st], (uint32_t)(j / STAGES) & 1, abort_flag, p.status);
+                __syncwarp();
+                named_bar_sync(BAR_P, BAR_P_COUNT);
+                if (lane == 0 && ok) {
+                    tc_fence_after();
+                    const uint64_t vd = sdesc_sw128(v0 + st * S::KV_BYTES, S::CHUNK, 1024);
+                    const uint32_t od = tmem_base + COL_O, pa = tmem_base + COL_S + (j & 1) * S_STRIDE;
+                    mma_f16_ts(od, pa, vd, IDESC_O, j > 0 ? 1u : 0u);
 #pragma unroll
-                        for (int kk = 1; kk < KT_ROWS / 16; ++kk) {
-                            // A = P from TMEM: 16 keys = 8 columns of fp16 pairs
-                            mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
-                        }
-                        mma_commit(&pv_done[st]);
-                    }
+                    for (int kk = 1; kk < KT_ROWS / 16; ++kk)
+                        mma_f16_ts(od, pa + kk * 8, sdesc_add(vd, kk * 16 * 128), IDESC_O, 1u);
+                    mma_commit(&pv_done[st]);
                 }
             }
             if (lane == 0) {
@@ -259,7 +272,7 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
         for (int j = 0; j < n_tiles; ++j) {
             const int b = j & 1;
             // after a failed wait the warp keeps looping without work, so that it still
-            // passes every tile's P barrier with the MMA warp
+            // passes every tile's P barrier with the P.V issuer
             if (ok) ok = mbar_wait_warp(&s_full[b], (j >> 1) & 1, abort_flag, p.status);
             if (!ok) {
                 named_bar_sync(BAR_P, BAR_P_COUNT);
@@ -326,9 +339,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
                 l_run += l_even + l_odd;
             }
 
-            // O is rescaled only once P.V_{j-1} has finished accumulating into it; P_j itself
-            // goes into S buffer b, whose previous P (of tile j-2) was read by P.V_{j-2}
-            // before S_j was written (the MMAs run in issue order)
+            // O is rescaled only once P.V_{j-1} has finished accumulating into it (the wait finds
+            // pv_done[(j-1) % 3] in the right phase: S_j was issued after P.V_{j-2} completed, so
+            // P.V_{j-4} is complete too); P_j itself goes into S buffer b, whose previous P (of
+            // tile j-2) P.V_{j-2} had read before the S issuer wrote S_j
             if (j >= 1 && __any_sync(0xffffffffu, resc)) {
                 if (!mbar_wait_warp(&pv_done[(j - 1) % STAGES], (uint32_t)((j - 1) / STAGES) & 1, abort_flag,
                                     p.status)) {

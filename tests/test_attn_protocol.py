@@ -2,34 +2,37 @@
 (paper_2609_09768_gb300/csrc/attn.cu), run on the CPU under many random schedules.
 
 The kernel has one wait without a time limit: the named barrier through which the four
-softmax warps hand P_j to the MMA warp (bar.sync, five warps, once per key tile).  Its
+softmax warps hand P_j to the P.V issuer (bar.sync, five warps, once per key tile).  Its
 safety rests on every warp passing it exactly once per tile on every path, including
 after a bounded mbarrier wait has run out.  The model replays the kernel's warps as
 cooperative actors:
 
   producer   : for tile j, wait pv_done[j % 3] (P.V of tile j - 3 done), issue the TMA load
-               of K_j and V_j onto kv_full[j % 3]
-  MMA warp   : wait q_ready; per j: wait kv_full (tile j), issue S_j and commit s_full[j % 2];
-               then pass the P barrier for tile j - 1 and issue P.V_{j-1}, commit pv_done
+               of K_j and V_j onto kv_full[j % 3]; it may stall between any two steps
+  S issuer   : wait q_ready; per j: wait kv_full (tile j), then for j >= 2 pv_done of tile
+               j - 2 (P.V_{j-2} read the buffer S_j overwrites), issue S_j, commit s_full[j % 2]
+  P.V issuer : per j: wait kv_full (tile j), pass the P barrier for tile j, issue P.V_j,
+               commit pv_done[j % 3]
   softmax x4 : arrive q_ready; per j: wait s_full, compute, optionally wait pv_done of tile
                j - 1 and rescale O, write P_j over S_j's buffer, pass the P barrier; finally
                wait pv_done of the last tile
 
-with the tensor pipe executing MMAs and commits in issue order, TMA loads landing after
-random delays, and mbarrier waits given parity semantics and a time limit that, when it
-runs out, sets the CTA's abort flag (every later incomplete wait then returns at once).
+Each issuer's MMAs run in its own issue order; the two issuers' MMAs are either not
+ordered with each other at all (two pipes running concurrently, the general case) or
+interleaved in one pipe.  TMA loads land after random delays, and mbarrier waits have
+parity semantics and a time limit that, when it runs out, sets the CTA's abort flag
+(every later incomplete wait then returns at once).
 
 Each run checks: every actor finishes (no deadlock, in particular at the P barrier); no
 warp arrives twice in one phase of the named barrier; no parity wait ever finds its
 barrier two phases ahead, nor asks for a phase while the one before it is still open
 (either would make the hardware answer wrongly: a parity wait cannot tell phase k from
-k - 2); and, in runs
-where no wait runs out, the data hazards are ordered: a slot is reloaded only after the
-P.V that read it, S_j runs only after K_j landed, P.V_j only after all four warps wrote
-P_j, S_{j+2} only after P.V_j read P_j from the same buffer, and O is rescaled only when
-no P.V into it is outstanding.  After a wait has run out the kernel still finishes but
-may compute on stale data in shared and tensor memory; it stays in bounds and the
-status word reports the timeout.
+k - 2); and, in runs where no wait runs out, the data hazards are ordered: a slot is
+reloaded only after the P.V that read it, S_j runs only after K_j landed and P.V_j only
+after V_j landed, P.V_j only after all four warps wrote P_j, S_{j+2} only after P.V_j read
+P_j from the same buffer, and O is rescaled only when no P.V into it is outstanding.
+After a wait has run out the kernel still finishes but may compute on stale data in
+shared and tensor memory; it stays in bounds and the status word reports the timeout.
 """
 import random
 
@@ -41,8 +44,9 @@ BAR_COUNT = N_SOFTMAX + 1
 
 
 class Protocol:
-    def __init__(self, n_tiles, seed, abort_at=None, limit=400):
+    def __init__(self, n_tiles, seed, abort_at=None, limit=400, shared_pipe=False):
         self.rng = random.Random(seed)
+        self.shared = shared_pipe        # one pipe for both issuers' MMAs, or one each
         self.n = n_tiles
         self.t = 0
         self.limit = limit               # ticks a bounded wait may last before it gives up
@@ -52,8 +56,8 @@ class Protocol:
         self.arrivals = {}               # (name, index) -> arrivals in the current phase
         self.expected = {("q_ready", 0): N_SOFTMAX}
         self.events = []                 # (tick, callable) for TMA completions
-        self.pipe = []                   # issued tensor-pipe work, in order
-        self.pipe_busy_until = 0
+        self.pipes = {"s": [], "pv": []}   # issued tensor-pipe work per issuer, in order
+        self.busy = {"s": 0, "pv": 0}
         self.bar_phase = 0
         self.bar_arrived = set()
         self.bar_waiting = set()
@@ -91,8 +95,13 @@ class Protocol:
             self.errors.append(f"{name}[{idx}] asked for phase {phase} while phase {c} is still open")
         return (c & 1) != parity
 
-    def issue(self, kind, j=None, commit=None):
-        self.pipe.append((kind, j, commit))
+    def issue(self, who, kind, j=None, commit=None):
+        self.pipes["s" if self.shared else who].append((kind, j, commit))
+
+    def stall(self):
+        """the producer may be slow to get to its next step"""
+        if self.rng.random() < 0.3:
+            yield ("delay", self.rng.randint(1, 80))
 
     # ------------------------------------------------------------------ actors
     def producer(self):
@@ -103,6 +112,7 @@ class Protocol:
                 break
             if j >= STAGES and (j - STAGES) not in self.done["PV"]:
                 self.hazard(f"slot {st} reloaded for tile {j} before P.V of tile {j - STAGES}")
+            yield from self.stall()
             delay = self.rng.randint(5, 60)
 
             def land(j=j, st=st):
@@ -110,18 +120,29 @@ class Protocol:
                 self.complete("kv_full", st)
             self.events.append((self.t + delay, land))
 
-    def mma(self):
+    def s_issuer(self):
         ok = yield ("wait", "q_ready", 0, 0, 0)
-        for j in range(self.n + 1):
-            if j < self.n and ok:
+        for j in range(self.n):
+            if not ok:
+                break
+            ok = yield ("wait", "kv_full", j % STAGES, (j // STAGES) & 1, j // STAGES)
+            if ok and j >= 2:
+                ok = yield ("wait", "pv_done", (j - 2) % STAGES, ((j - 2) // STAGES) & 1, (j - 2) // STAGES)
+            if not ok:
+                break
+            self.issue("s", "S", j, ("s_full", j % 2))
+        self.issue("s", "drain", None, ("drain_s", 0))
+        yield ("wait", "drain_s", 0, 0, 0)
+
+    def pv_issuer(self):
+        ok = True
+        for j in range(self.n):
+            if ok:
                 ok = yield ("wait", "kv_full", j % STAGES, (j // STAGES) & 1, j // STAGES)
-                if ok:
-                    self.issue("S", j, ("s_full", j % 2))
-            if j >= 1:
-                yield ("bar",)
-                if ok:
-                    self.issue("PV", j - 1, ("pv_done", (j - 1) % STAGES))
-        self.issue("drain", None, ("drain", 0))
+            yield ("bar",)
+            if ok:
+                self.issue("pv", "PV", j, ("pv_done", j % STAGES))
+        self.issue("pv", "drain", None, ("drain", 0))
         yield ("wait", "drain", 0, 0, 0)
 
     def softmax(self, w):
@@ -151,37 +172,41 @@ class Protocol:
             yield ("wait", "pv_done", (self.n - 1) % STAGES, ((self.n - 1) // STAGES) & 1, (self.n - 1) // STAGES)
 
     # ------------------------------------------------------------------ tensor pipe
-    def step_pipe(self):
-        if not self.pipe or self.t < self.pipe_busy_until:
+    def step_one(self, key):
+        q = self.pipes[key]
+        if not q or self.t < self.busy[key]:
             return False
-        kind, j, commit = self.pipe.pop(0)
-        if kind == "S":
-            if j not in self.done["kv"]:
-                self.hazard(f"S_{j} ran before K_{j} landed")
-            if j >= 2 and (j - 2) not in self.done["PV"]:
-                self.hazard(f"S_{j} overwrote P_{j - 2} before P.V_{j - 2} read it")
-        if kind == "PV":
-            if self.p_written.get(j, set()) != set(range(N_SOFTMAX)):
-                self.hazard(f"P.V_{j} ran before all warps wrote P_{j}")
-        self.pipe_busy_until = self.t + (self.rng.randint(4, 12) if kind != "drain" else 0)
+        kind, j, commit = q.pop(0)
+        if kind in ("S", "PV") and j not in self.done["kv"]:
+            self.hazard(f"{kind}_{j} ran before K_{j} and V_{j} landed")
+        if kind == "S" and j >= 2 and (j - 2) not in self.done["PV"]:
+            self.hazard(f"S_{j} overwrote P_{j - 2} before P.V_{j - 2} read it")
+        if kind == "PV" and self.p_written.get(j, set()) != set(range(N_SOFTMAX)):
+            self.hazard(f"P.V_{j} ran before all warps wrote P_{j}")
+        self.busy[key] = self.t + (self.rng.randint(4, 12) if kind != "drain" else 0)
 
         def finish(kind=kind, j=j, commit=commit):
             if kind in ("S", "PV"):
                 self.done[kind].add(j)
             if commit:
                 self.complete(*commit)
-        self.events.append((self.pipe_busy_until, finish))
+        self.events.append((self.busy[key], finish))
         return True
+
+    def step_pipe(self):
+        a = self.step_one("s")
+        b = self.step_one("pv")
+        return a or b
 
     # ------------------------------------------------------------------ scheduler
     def run(self, max_ticks=200000):
-        actors = {"producer": self.producer(), "mma": self.mma()}
+        actors = {"producer": self.producer(), "s_issuer": self.s_issuer(), "pv_issuer": self.pv_issuer()}
         for w in range(N_SOFTMAX):
             actors[f"softmax{w}"] = self.softmax(w)
         state = {}                       # actor -> (request, start tick)
         values = {a: None for a in actors}
         finished = set()
-        bar_members = {"mma"} | {f"softmax{w}" for w in range(N_SOFTMAX)}
+        bar_members = {"pv_issuer"} | {f"softmax{w}" for w in range(N_SOFTMAX)}
         while len(finished) < len(actors):
             if self.t > max_ticks:
                 raise AssertionError(f"deadlock: waiting {sorted(set(actors) - finished)} at tick {self.t}")
@@ -240,26 +265,28 @@ class Protocol:
         return self.bar_phase
 
 
+@pytest.mark.parametrize("shared_pipe", [False, True])
 @pytest.mark.parametrize("n_tiles", [1, 2, 3, 4, 7, 20])
-def test_protocol_completes_and_orders_every_hazard(n_tiles):
+def test_protocol_completes_and_orders_every_hazard(n_tiles, shared_pipe):
     for seed in range(40):
-        phases = Protocol(n_tiles, seed).run()
+        phases = Protocol(n_tiles, seed, shared_pipe=shared_pipe).run()
         assert phases == n_tiles                      # one P-barrier phase per key tile
 
 
+@pytest.mark.parametrize("shared_pipe", [False, True])
 @pytest.mark.parametrize("n_tiles", [1, 3, 6, 20])
-def test_protocol_completes_after_a_wait_runs_out(n_tiles):
+def test_protocol_completes_after_a_wait_runs_out(n_tiles, shared_pipe):
     """Some wait gives up at a random tick: every warp still passes every tile's P
     barrier once, so the barrier cannot block the kernel's exit."""
     for seed in range(60):
         rng = random.Random(1000 + seed)
-        phases = Protocol(n_tiles, seed, abort_at=rng.randint(0, 40 * n_tiles)).run()
+        phases = Protocol(n_tiles, seed, abort_at=rng.randint(0, 40 * n_tiles), shared_pipe=shared_pipe).run()
         assert phases == n_tiles
 
 
 def test_model_catches_a_warp_that_skips_the_barrier():
-    """The check has teeth: a softmax warp that leaves its loop after a failed wait (the
-    kernel's behaviour before the named barrier) leaves the MMA warp blocked."""
+    """The check has teeth: a softmax warp that leaves its loop after a failed wait leaves
+    the P.V issuer blocked at the barrier."""
     class Skipping(Protocol):
         def softmax(self, w):
             self.arrive("q_ready", 0)
@@ -293,11 +320,32 @@ def test_model_catches_a_slot_reloaded_too_early():
         Eager(12, 0).run()
 
 
+def test_model_catches_s_issued_before_the_pv_that_reads_its_buffer():
+    """The two issuers' MMAs are not ordered with each other, so an S issuer that does not
+    wait for P.V_{j-2} can overwrite P_{j-2} before it is read."""
+    class NoPvWait(Protocol):
+        def s_issuer(self):
+            yield ("wait", "q_ready", 0, 0, 0)
+            for j in range(self.n):
+                yield ("wait", "kv_full", j % STAGES, (j // STAGES) & 1, j // STAGES)
+                self.issue("s", "S", j, ("s_full", j % 2))
+            self.issue("s", "drain", None, ("drain_s", 0))
+            yield ("wait", "drain_s", 0, 0, 0)
+    caught = 0
+    for seed in range(10):
+        try:
+            NoPvWait(12, seed).run()
+        except AssertionError as e:
+            assert "overwrote" in str(e) or "two phases" in str(e) or "still open" in str(e), e
+            caught += 1
+    assert caught >= 8
+
+
 def test_model_catches_a_wait_on_a_phase_not_yet_reached():
-    """A producer that frees slot j % 3 by waiting for S_{j-1} (issued after P.V_{j-3}, so
-    done after it in a single in-order pipe) on the double-buffered s_full barrier asks,
-    at tiles 3 and 4, for a phase the barrier has not reached while the one before is still
-    open; the hardware answers such a parity wait at once.  The model flags it."""
+    """A producer that frees slot j % 3 by waiting for S_{j-1} on the double-buffered
+    s_full barrier asks, at tiles 3 and 4, for a phase the barrier has not reached while
+    the one before is still open; the hardware answers such a parity wait at once.  The
+    model flags it."""
     class WaitsOnS(Protocol):
         def producer(self):
             for j in range(self.n):
@@ -313,3 +361,4 @@ def test_model_catches_a_wait_on_a_phase_not_yet_reached():
                 self.events.append((self.t + 5, land))
     with pytest.raises(AssertionError, match="still open"):
         WaitsOnS(12, 0).run()
+
