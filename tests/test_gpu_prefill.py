@@ -238,6 +238,43 @@ def test_single_chunk_is_exact_for_any_ratio(kvb):
         print("single chunk r", r, e)
 
 
+def test_context_cache_does_not_depend_on_the_query(kvb, case):
+    """The same request without its query suffix: HKVD compares context rows only and every
+    recomputed row attends keys at or before its own position, so the selection and the
+    context rows of the blended cache are bit-identical (a block whose key range grows
+    because it also holds query rows only adds fully masked tiles, which contribute zero)."""
+    ck, cv = case.new_cache()
+    _, sel, _ = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, case.dtoks,
+                                      case.dstarts, case.n_ctx, case.nq, case.wl.r, 1, ws=case.ws)
+    ck0, cv0 = case.new_cache()
+    fh0, sel0, t0 = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck0, cv0,
+                                          case.dtoks[: case.n_ctx], case.dstarts, case.n_ctx, 0, case.wl.r, 1,
+                                          ws=case.ws, timings=True)
+    torch.cuda.synchronize()
+    assert kvb.device_status(case.ws) == 0
+    k = blend.num_selected(case.wl.r, case.n_ctx)
+    assert fh0.shape[0] == 0 and t0["n_selected"] == k and t0["n_rows"] == k
+    assert torch.equal(sel[:k], sel0[:k])
+    n = case.n_ctx
+    assert torch.equal(ck[:, :n], ck0[:, :n]) and torch.equal(cv[:, :n], cv0[:, :n])
+
+
+def test_query_only_request_is_a_dense_prefill(kvb, case):
+    """No cached context: nothing to merge or select, so the call is the dense prefill of the
+    query tokens, bit for bit."""
+    q = case.dtoks[case.n_ctx:].clone()      # a fresh buffer: the call wants 16-byte aligned token ids
+    ck, cv = case.new_cache()
+    fh, _, t = kvb.selective_prefill(case.cfg, case.model, case.rope, case.kch, case.vch, ck, cv, q, case.dstarts,
+                                     0, case.nq, case.wl.r, 1, ws=case.ws, timings=True)
+    ck2, cv2 = case.new_cache()
+    fh2, _ = kvb.full_prefill(case.cfg, case.model, case.rope, ck2, cv2, q, n_out=case.nq, ws=case.ws)
+    torch.cuda.synchronize()
+    assert kvb.device_status(case.ws) == 0
+    assert t["n_selected"] == 0
+    assert torch.equal(fh, fh2)
+    assert torch.equal(ck[:, : case.nq], ck2[:, : case.nq]) and torch.equal(cv[:, : case.nq], cv2[:, : case.nq])
+
+
 def test_repeatable_bitwise(kvb, case):
     """Three runs on the same inputs give bit-identical outputs (no races in the pipeline)."""
     outs = []
