@@ -37,7 +37,7 @@ METRIC = "TTFT (ms) at 124k tokens r=0.15 vs own r=1.0 prefill; attn TFLOP/s, % 
 # size (18,713 rows over a 124,032-row cache), from one ncu capture of that launch; valid
 # only for the kernel sources it was taken on (sha1 prefixes of attn.cu and common.cuh),
 # otherwise reported as null.
-ATTN_TRAFFIC = {"bytes": 8.162245e9 + 0.141590e9, "sha1": {"attn.cu": "7960fd435f01", "common.cuh": "ac1f1dda7832"}}
+ATTN_TRAFFIC = {"bytes": 0.878205e9 + 0.142111e9, "sha1": {"attn.cu": "0b224fed4482", "common.cuh": "ac1f1dda7832"}}
 
 
 def attn_traffic():

@@ -1,6 +1,8 @@
 // Sparse-query causal GQA flash attention on the 5th-generation tensor cores.
 //
-// Each CTA owns one (block of query rows, kv head) unit.  The G = Hq/Hkv query heads
+// Each CTA owns one (block of query rows, kv head) unit; units are numbered kv head
+// major, heaviest row block first within a head, so that the CTAs resident at a time read
+// the K/V of one or two kv heads (63 MB each at 124k keys), which L2 holds.  The G = Hq/Hkv query heads
 // that share kv head g are packed with RPB = floor(128/G) query rows into the 128
 // rows of one MMA tile (lane = row_in_block * G + head_in_group; the last 128 - RPB*G
 // lanes idle when G does not divide 128), so every K/V tile loaded serves all G heads.
@@ -105,8 +107,10 @@ attn_kernel(const uint16_t* __restrict__ q, const __grid_constant__ CUtensorMap 
     const uint32_t warp = warp_id(), lane = lane_id();
     const int G = p.Hq / p.Hkv;
     const int RPB = 128 / G;
-    const int blk = num_blocks - 1 - (int)(blockIdx.x / p.Hkv);   // heaviest rows first
-    const int g = (int)(blockIdx.x % p.Hkv);
+    // kv head major (the CTAs resident at a time read one or two heads' K/V, which L2 holds),
+    // heaviest rows first within a head
+    const int blk = num_blocks - 1 - (int)(blockIdx.x % num_blocks);
+    const int g = (int)(blockIdx.x / num_blocks);
     const int64_t r0 = (int64_t)blk * RPB;
 
     if (threadIdx.x == 0) {
