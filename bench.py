@@ -216,6 +216,12 @@ class OracleSample:
         return (t1 - t0) + (t3 - t2), t2 - t1
 
 
+def sample_rows(args, wl, k: int) -> int:
+    """Rows in the oracle's timed sample: --cpu-rows within [16, 256], and no more than the
+    rows the method recomputes (k + n_query) or the context holds."""
+    return max(1, min(max(16, min(256, args.cpu_rows)), k + wl.n_query, wl.n_ctx))
+
+
 def cpu_cores() -> int:
     try:
         return len(os.sched_getaffinity(0))
@@ -247,7 +253,7 @@ def run_reference(args, wl, rank: int, world: int) -> None:
     from oracle import blend
     r = wl.r if args.r is None else args.r
     k = blend.num_selected(r, wl.n_ctx)
-    rows = max(16, min(256, args.cpu_rows))
+    rows = sample_rows(args, wl, k)
     smp = OracleSample(wl, rows)
     for _ in range(args.warmup):
         smp.run()
@@ -516,7 +522,7 @@ def run_ours(args, wl, rank: int, world: int) -> None:
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        n = max(16, min(256, args.cpu_rows))
+        n = sample_rows(args, wl, k)
         smp = OracleSample(wl, n)
         t_rows, t_attn = smp.run()
         sel_np = sel[:k].cpu().numpy() if k > 0 else None
