@@ -17,7 +17,10 @@ bf16 ulp of the value per element (plus 2e-2 of the RMS) and mean-abs <= 2e-3 of
 The layer outputs: max-abs <= 2e-2 and mean-abs <= 2e-3 of the output's RMS, against the
 float64 oracle with the bf16 storage points of the paper's bf16 model and against the
 oracle's float32-accumulation run (the literal fp32 oracle).  The stated bar in absolute
-units is reported for every layer beside the distance between the two oracles themselves:
+units is asserted from layer 2 on (layers 15 and 31 of the 32-layer stacks) and reported for
+layers 0 and 1 beside the distance between the two oracles themselves: at the first two
+layers it lies within what fp32-level changes alone move the output
+(tests/test_precision_floor.py), for this reason:
 the residual rows have an RMS of 2.6 after layer 0 and grow with depth, and a perturbation
 of one part in 10^7 before a bf16 rounding (an RMSNorm output, the attention output)
 flips that rounding now and then; through the 4096 -> 14336 fan-out of the MLP a few
@@ -144,8 +147,10 @@ def _check_layer(run, l, smp, what):
     ek = assert_close_bf16(k_gpu.reshape(len(pos), -1), kv["fp64"][0], f"{what} layer {l} K")
     ev = assert_close_bf16(v_gpu.reshape(len(pos), -1), kv["fp64"][1], f"{what} layer {l} V")
     print(f"{what} layer {l}: K {ek}, V {ev}")
-    # layer output: the stated bar relative to the output's RMS (the absolute form is reported above)
+    # layer output: the stated bar relative to the output's RMS, and in absolute units from layer 2 on
     assert_close_rel(x_out, outs["fp64"], f"{what} layer {l} output vs fp64 oracle")
+    if l >= 2:
+        assert absolute, f"{what} layer {l} output vs fp64 oracle, absolute bar: {e64}"
     assert_close_rel(x_out, outs["fp32acc"], f"{what} layer {l} output vs fp32-accumulation oracle")
     return dict(e64=e64, e32=e32, floor=floor, absolute=absolute)
 
