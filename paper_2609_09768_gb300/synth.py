@@ -146,6 +146,8 @@ WORKLOADS: Dict[str, Workload] = {
     "l8b_1layer": Workload("llama8b-2L-8x480+64", LLAMA8B.with_layers(2), 8, 480, 64),
     "l8b_32k": Workload("llama8b-32L-64x512+128", LLAMA8B, 64, 512, 128),
     "l8b_124k": Workload("llama8b-32L-242x512+128", LLAMA8B, 242, 512, 128),
+    # the 64k-context request of the r x chunk-size sweep, at its largest chunks and r = 0.25
+    "l8b_64k": Workload("llama8b-32L-32x2048+128", LLAMA8B, 32, 2048, 128, r=0.25),
     # two special tokens between documents, their cache rows zero
     "tiny_sep": Workload("tiny-2L-4x126+sep2+32", TINY, 4, 126, 32, n_sep=2),
     "l8b_1layer_sep": Workload("llama8b-2L-8x478+sep2+64", LLAMA8B.with_layers(2), 8, 478, 64, n_sep=2),

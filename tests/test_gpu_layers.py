@@ -1,6 +1,7 @@
 """Per-layer parity of the selective prefill, teacher-forced, on the Llama-3.1-8B-shaped
 workloads: the 2-layer model (3.9k tokens) and the 32-layer stacks at 32.9k tokens
-(64 x 512 + 128) and 124k tokens (242 x 512 + 128, the headline request); and on the
+(64 x 512 + 128), 65.7k tokens (32 x 2048 + 128 at r = 0.25, the context of the r x
+chunk-size sweep) and 124k tokens (242 x 512 + 128, the headline request); and on the
 32-layer YaRN model with seven q heads per kv head and a q/k/v bias at 124k tokens.
 
 One call of kvb_selective_prefill runs the whole path; layer taps capture the residual
@@ -159,7 +160,7 @@ def _check_layer(run, l, smp, what):
 _RUNS = {}
 
 
-@pytest.fixture(scope="module", params=["l8b_1layer", "l8b_32k", "l8b_124k", "yarn_124k"])
+@pytest.fixture(scope="module", params=["l8b_1layer", "l8b_32k", "l8b_64k", "l8b_124k", "yarn_124k"])
 def run(request, kvb):
     # one workload resident at a time (the 124k one holds ~40 GB of caches and weights)
     for key in list(_RUNS):
